@@ -1,0 +1,518 @@
+"""Throughput of the pooled embedding-bag forward + de-duplicated backward on GB300.
+
+One step = the whole hot path on one batch: forward gather-pool, then the
+backward (key generation, radix sort, run-length pass, segmented reduce).
+Prints one JSON line (rank 0). Defaults: 1 GPU, the 128 GB workload cfg5.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload cfg5]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on a bounded sample
+
+Under torchrun every rank runs an independent replica (its own tables and
+batches; no collective on the data path) and rank 0 reports the whole-job
+throughput: all ranks' bytes over the slowest rank's time ("weak" scaling).
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2609_30656_gb300 import metrics, workloads as wl  # noqa: E402
+
+METRIC = "embedding-bag fwd/bwd HBM GB/s and % of GB300 peak; rows gathered/sec"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def measured_hbm_peak() -> tuple[float, str]:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def describe(w: wl.Workload) -> str:
+    L = w.lengths
+    if L.kind == "fixed":
+        lens = f"every bag {int(L.mean)} long"
+    elif L.kind == "poisson":
+        lens = f"Poisson({L.mean:g}) lengths clipped to [{L.lo}, {L.hi}]"
+    elif L.kind == "lognormal":
+        lens = f"lognormal lengths (mean {L.mean:g}, max {L.hi})"
+    else:
+        lens = (f"{L.empty_frac:.0%} empty bags, others power law L^-{L.alpha:g} on "
+                f"[{L.lo}, {L.hi}]")
+    idx = "uniform indices" if w.zipf_alpha is None else f"Zipf({w.zipf_alpha:g}) indices"
+    pool = ("weighted " if w.weighted else "") + ("mean" if w.mean else "sum")
+    rows = (f"{w.num_tables} x {w.rows[0]:,} rows" if len(set(w.rows)) == 1
+            else f"{w.num_tables} tables, {min(w.rows):,}..{max(w.rows):,} rows")
+    dims = "/".join(str(d) for d in sorted(set(w.dims)))
+    return (f"{w.name}: {rows} x dim {dims} {w.dtype}, batch {w.batch}, {lens}, {idx}, {pool} "
+            f"pooling, forward + de-duplicated backward")
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_30656_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if taken on this source."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    entry = rec.get(workload, {}).get(kernel)
+    if not entry or entry.get("source_hash") != kernel_source_hash():
+        return None
+    return entry.get("bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.3)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) != 7:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), float(parts[2]), parts[3:]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, _, flags in rows for i, fl in enumerate(flags)
+                          if fl.lower().startswith("active")})
+        loaded = [r for r in rows if r[2] > 200.0] or rows
+        return {"sm_mhz": statistics.median(r[0] for r in loaded),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(r[2] for r in rows)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def aggregate(local_ms: float, local_bytes: float, local_rows: float, world: int):
+    """Max time and summed work over ranks (identity at world size 1)."""
+    if world == 1 or not torch.distributed.is_initialized():
+        return local_ms, local_bytes, local_rows
+    dev = torch.device("cuda", torch.cuda.current_device()) if torch.cuda.is_available() and \
+        torch.distributed.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([local_ms], dtype=torch.float64, device=dev)
+    s = torch.tensor([local_bytes, local_rows], dtype=torch.float64, device=dev)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    torch.distributed.all_reduce(s, op=torch.distributed.ReduceOp.SUM)
+    return float(t[0]), float(s[0]), float(s[1])
+
+
+# ----------------------------------------------------------------------------- oracle leg
+
+def _compact(tables, indices, offsets, weights, batch, tabs_idx):
+    """Host copies of the rows touched by the chosen tables, indices renumbered."""
+    host_tabs, host_ind, off_parts, w_parts = [], [], [], []
+    lens = []
+    for t in tabs_idx:
+        s, e = int(offsets[t * batch]), int(offsets[(t + 1) * batch])
+        idx = indices[s:e]
+        uniq = torch.unique(idx)
+        host_tabs.append(tables[t].index_select(0, uniq).cpu())
+        host_ind.append(torch.searchsorted(uniq, idx).cpu())
+        lens.append((offsets[t * batch + 1:(t + 1) * batch + 1] -
+                     offsets[t * batch:(t + 1) * batch]).cpu())
+        if weights is not None:
+            w_parts.append(weights[s:e].cpu())
+    L = torch.cat(lens)
+    off = torch.zeros(L.numel() + 1, dtype=torch.int64)
+    off[1:] = torch.cumsum(L, 0)
+    ind = torch.cat(host_ind) if host_ind else torch.zeros(0, dtype=torch.int64)
+    w = torch.cat(w_parts) if weights is not None else None
+    return host_tabs, ind, off, w
+
+
+def oracle_step(host_tabs, ind, off, w, go, batch, mean, threads):
+    import numpy as np
+
+    import oracle
+    t0 = time.perf_counter()
+    oracle.forward(host_tabs, batch, ind, off, weights=w, mean=mean, threads=threads)
+    rows = np.array([t.shape[0] for t in host_tabs], np.int64)
+    dims = np.array([t.shape[1] for t in host_tabs], np.int32)
+    res = oracle.backward(rows, dims, batch, ind, off, go, weights=w, mean=mean, threads=threads)
+    return time.perf_counter() - t0, res
+
+
+def sample_problem(w, tables, batch0, go0, num_tables):
+    tabs_idx = list(range(num_tables))
+    host_tabs, ind, off, wt = _compact(tables, batch0.indices, batch0.offsets, batch0.weights,
+                                       w.batch, tabs_idx)
+    dims = [w.dims[t] for t in tabs_idx]
+    cols = []
+    for t in tabs_idx:
+        d0 = sum(w.dims[:t])
+        cols.append(go0[:, d0:d0 + w.dims[t]])
+    go = torch.cat(cols, dim=1).cpu().contiguous()
+    counts = metrics.batch_counts(dims, w.elem_bytes, w.batch, off, wt is not None)
+    return host_tabs, ind, off, wt, go, counts
+
+
+def sample_bytes(counts, res, rows_of_tables):
+    toff = res.table_offsets
+    uniq = [int(toff[i + 1] - toff[i]) for i in range(len(toff) - 1)]
+    return metrics.forward_bytes(counts)["total"] + metrics.backward_bytes(counts, uniq)["total"]
+
+
+def cpu_threads() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_ours(args):
+    import numpy as np
+
+    from paper_2609_30656_gb300 import tbe
+
+    world, rank, local = dist_env()
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = wl.get_workload(args.workload)
+    seed = args.seed
+    tables = wl.make_tables(w, seed, dev)
+    batches = [wl.make_batch(w, seed + 1000 * rank, dev, batch_index=k) for k in range(args.rotate)]
+    grads_out = [wl.make_grad_out(w, seed + 1000 * rank, dev, batch_index=k)
+                 for k in range(args.rotate)]
+    m = tbe.TBE(tables, pooling="mean" if w.mean else "sum", timing=True)
+    max_n = max(b.num_indices for b in batches)
+    m.reserve(w.batch, max_n)
+    out = torch.empty(w.batch, w.sum_dims, dtype=torch.float32, device=dev)
+    # Size the sparse gradient from a counting pass over every rotating batch.
+    U_max, F_max, uniq_tables = 0, 0, []
+    for b, go in zip(batches, grads_out):
+        probe = m.alloc_grad(0, 0, size_only=True)
+        m.backward_into(probe, b.indices, b.offsets, go, b.weights)
+        U_max = max(U_max, probe.num_unique)
+        F_max = max(F_max, probe.num_floats)
+        toff = probe.table_offsets.cpu().tolist()
+        uniq_tables.append([toff[t + 1] - toff[t] for t in range(w.num_tables)])
+    g = m.alloc_grad(U_max, F_max)
+    counts = [metrics.batch_counts(w.dims, w.elem_bytes, w.batch, b.offsets, b.weights is not None)
+              for b in batches]
+    packed = w.weighted or w.mean
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev)
+
+    def step(k):
+        b, go = batches[k % args.rotate], grads_out[k % args.rotate]
+        m.forward(b.indices, b.offsets, b.weights, out=out)
+        m.backward_into(g, b.indices, b.offsets, go, b.weights)
+
+    for k in range(args.warmup):
+        step(k)
+    if m.get_error() != 0:
+        raise RuntimeError("device-side error during warm-up")
+    torch.cuda.synchronize()
+
+    names = tbe.component_names()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    comp = {n: [] for n in names}
+    launches0 = m.launch_count()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        wall0 = time.perf_counter()
+        for k in range(args.steps):
+            flush.zero_()  # L2 starts cold each step (outside the step's events)
+            starts[k].record()
+            step(args.warmup + k)
+            stops[k].record()
+            for n_, v in m.last_timings().items():
+                comp[n_].append(v)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+    if world > 1:
+        torch.distributed.barrier()
+    launches = m.launch_count() - launches0
+    if m.get_error() != 0:
+        raise RuntimeError("device-side error during the timed steps")
+    step_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
+    ms = sum(step_ms) / len(step_ms)
+
+    # Work of the timed steps (host-side sizes).
+    fwd_b, bwd_b, rows_g = 0.0, 0.0, 0.0
+    comp_bytes = {n: 0.0 for n in names}
+    uniq_fwd = 0.0
+    for k in range(args.steps):
+        i = (args.warmup + k) % args.rotate
+        c = counts[i]
+        fwd_b += metrics.forward_bytes(c)["total"]
+        bwd_b += metrics.backward_bytes(c, uniq_tables[i])["total"]
+        uniq_fwd += metrics.forward_unique_bytes(c, uniq_tables[i])
+        rows_g += 2 * c.n
+        for n_, v in metrics.component_bytes(c, uniq_tables[i], w.rows, packed).items():
+            comp_bytes[n_] += v
+    per_step_bytes = (fwd_b + bwd_b) / args.steps
+    tot_ms, tot_bytes, tot_rows = aggregate(ms, per_step_bytes, rows_g / args.steps, world)
+    gbs = tot_bytes / (tot_ms * 1e-3) / 1e9
+    peak, peak_kind = measured_hbm_peak()
+
+    comp_ms = {n: statistics.mean(v) for n, v in comp.items() if v and min(v) >= 0}
+    fwd_ms = comp_ms["fwd.prep"] + comp_ms["fwd.gather"] + comp_ms["fwd.fixup"]
+    bwd_ms = sum(comp_ms[n] for n in names if n.startswith("bwd."))
+    components = {}
+    for n in names:
+        if n not in comp_ms:
+            continue
+        cb = comp_bytes.get(n)
+        entry = {"ms": round(comp_ms[n], 4), "share": round(comp_ms[n] / (fwd_ms + bwd_ms), 4)}
+        if cb:
+            entry["alg_gbs"] = round(cb / args.steps / (comp_ms[n] * 1e-3) / 1e9, 1)
+        components[n] = entry
+    dominant = max((n for n in comp_bytes if n in comp_ms), key=lambda n: comp_ms[n])
+    dom_bytes = comp_bytes[dominant] / args.steps
+    achieved = dom_bytes / (comp_ms[dominant] * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "kernel": dominant, "achieved": round(achieved, 1),
+                "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+                else "fallback 6800 GB/s",
+                "traffic": recorded_traffic(dominant, w.name),
+                "bytes_per_launch": int(dom_bytes)}
+    mean_counts_n = statistics.mean(c.n for c in counts)
+    fwd_bytes_step = fwd_b / args.steps
+    bwd_bytes_step = bwd_b / args.steps
+    line = {
+        "metric": METRIC, "value": round(gbs, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(tot_ms, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "storage_dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": describe(w),
+                   "l2": f"flushed before every step ({2 * l2 >> 20} MB write, outside the "
+                         "step's events); inputs also exceed L2",
+                   "rotating_batches": args.rotate, "seed": seed,
+                   "lookups_per_step": int(mean_counts_n), "parallelism": f"replicas x{world}"},
+        "pct_hbm": round(gbs / world / peak, 4), "pct_hbm_nominal": round(gbs / world / NOMINAL_HBM_GBS, 4),
+        "rows_per_s": round(tot_rows / (tot_ms * 1e-3), 1),
+        "fwd": {"ms": round(fwd_ms, 4), "alg_gbs": round(fwd_bytes_step / (fwd_ms * 1e-3) / 1e9, 1),
+                "pct_hbm": round(fwd_bytes_step / (fwd_ms * 1e-3) / 1e9 / peak, 4),
+                "rows_per_s": round(mean_counts_n / (fwd_ms * 1e-3), 1),
+                "unique_row_gbs": round(uniq_fwd / args.steps / (fwd_ms * 1e-3) / 1e9, 1)},
+        "bwd": {"ms": round(bwd_ms, 4), "alg_gbs": round(bwd_bytes_step / (bwd_ms * 1e-3) / 1e9, 1),
+                "pct_hbm": round(bwd_bytes_step / (bwd_ms * 1e-3) / 1e9 / peak, 4),
+                "rows_per_s": round(mean_counts_n / (bwd_ms * 1e-3), 1)},
+        "components": components,
+        "roofline": roofline,
+        "gpu_launches": int(launches),
+        "wall_ms_per_step": round(wall * 1e3 / args.steps, 3),
+        "clocks": clk.summary(),
+    }
+
+    # End to end through the public API from pinned host memory.
+    if not args.no_e2e:
+        line["e2e"] = run_e2e(args, m, w, batches, grads_out, g, out, dev, world)
+    # The oracle on the host cores, rank 0 only, single GPU runs only.
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = run_cpu_baseline(args, w, tables, batches[0], grads_out[0])
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_e2e(args, m, w, batches, grads_out, g, out, dev, world):
+    b, go = batches[0], grads_out[0]
+    h_ind = b.indices.cpu().pin_memory()
+    h_off = b.offsets.cpu().pin_memory()
+    h_w = None if b.weights is None else b.weights.cpu().pin_memory()
+    h_go = go.cpu().pin_memory()
+    h_res = torch.empty(2 + w.num_tables + 1, dtype=torch.int64).pin_memory()
+    steps = max(2, min(args.steps, args.e2e_steps))
+    bytes_in = (h_ind.numel() * 8 + h_off.numel() * 8 + (0 if h_w is None else h_w.numel() * 4)
+                + h_go.numel() * 4)
+    bytes_out = h_res.numel() * 8
+
+    def e2e_step():
+        # The user's call: host batch and upstream gradient in, step result out.
+        y = m.forward(h_ind, h_off, h_w, out=out)
+        m.backward_into(g, h_ind, h_off, h_go, h_w)
+        h_res[0:1].copy_(g.num_unique_dev, non_blocking=True)
+        h_res[1:2].copy_(g.num_floats_dev, non_blocking=True)
+        h_res[2:].copy_(g.table_offsets, non_blocking=True)
+        return y
+
+    e2e_step()
+    torch.cuda.synchronize()
+    counts = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, b.offsets, b.weights is not None)
+    toff = g.table_offsets.cpu().tolist()
+    uniq = [toff[t + 1] - toff[t] for t in range(w.num_tables)]
+    step_bytes = metrics.forward_bytes(counts)["total"] + metrics.backward_bytes(counts, uniq)["total"]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    el = (time.perf_counter() - t0) / steps
+    tot_ms, tot_bytes, _ = aggregate(el * 1e3, step_bytes, 0.0, world)
+    return {"value": round(tot_bytes / (tot_ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+            "ms_per_step": round(tot_ms, 3), "steps": steps,
+            "h2d_bytes_per_step": int(bytes_in), "d2h_bytes_per_step": int(bytes_out),
+            "note": "host batch (indices, offsets, weights) and grad_out copied from pinned "
+                    "memory by the binding each step; num_unique, num_floats and table_offsets "
+                    "read back"}
+
+
+def run_cpu_baseline(args, w, tables, batch0, go0, budget_s: float | None = None):
+    threads = cpu_threads()
+    ntab = min(w.num_tables, args.cpu_tables)
+    host_tabs, ind, off, wt, go, counts = sample_problem(w, tables, batch0, go0, ntab)
+    el, res = oracle_step(host_tabs, ind, off, wt, go, w.batch, w.mean, threads)
+    nbytes = sample_bytes(counts, res, w.rows[:ntab])
+    return {"value": round(nbytes / el / 1e9, 3), "unit": "GB/s", "cores": threads,
+            "kind": "oracle",
+            "sample": f"forward + backward of tables 0..{ntab - 1} of {w.num_tables} at the full "
+                      f"batch ({counts.n:,} lookups, {nbytes / 1e9:.2f} GB algorithmic), "
+                      f"{el:.1f} s on {threads} threads (OpenMP over bags; the sort is serial)"}
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return  # rank 0 alone times the oracle
+    dev = torch.device("cuda", 0) if torch.cuda.is_available() else torch.device("cpu")
+    w = wl.get_workload(args.workload)
+    threads = cpu_threads()
+    ntab = min(w.num_tables, args.ref_tables)
+    tables = wl.make_tables(w, args.seed, dev, only=range(ntab))
+    b = wl.make_batch(w, args.seed, dev)
+    go = wl.make_grad_out(w, args.seed, dev)
+    host_tabs, ind, off, wt, gos, counts = sample_problem(w, tables, b, go, ntab)
+    # Shrink the sample (batch rows) so the whole run stays within a few minutes.
+    el, res = oracle_step(host_tabs, ind, off, wt, gos, w.batch, w.mean, threads)
+    budget = args.ref_budget_s / max(1, args.steps + args.warmup)
+    frac = min(1.0, budget / max(el, 1e-6))
+    keep_b = max(64, int(w.batch * frac))
+    if keep_b < w.batch:
+        L = (off[1:] - off[:-1]).view(ntab, w.batch)[:, :keep_b]
+        new_off = torch.zeros(ntab * keep_b + 1, dtype=torch.int64)
+        new_off[1:] = torch.cumsum(L.reshape(-1), 0)
+        keep = torch.cat([torch.arange(int(off[t * w.batch]), int(off[t * w.batch]) + int(L[t].sum()))
+                          for t in range(ntab)])
+        ind, off = ind[keep], new_off
+        wt = None if wt is None else wt[keep]
+        gos = gos[:keep_b].contiguous()
+        counts = metrics.batch_counts([w.dims[t] for t in range(ntab)], w.elem_bytes, keep_b, off,
+                                      wt is not None)
+    times, nb = [], 0
+    for k in range(args.warmup + args.steps):
+        el, res = oracle_step(host_tabs, ind, off, wt, gos, keep_b, w.mean, threads)
+        if k >= args.warmup:
+            times.append(el)
+            nb = sample_bytes(counts, res, w.rows[:ntab])
+    ms = statistics.mean(times) * 1e3
+    gbs = nb / (ms * 1e-3) / 1e9
+    sample = (f"forward + backward of tables 0..{ntab - 1} of {w.num_tables}, first {keep_b} of "
+              f"{w.batch} batch rows ({counts.n:,} lookups, {nb / 1e9:.3f} GB algorithmic)")
+    line = {"impl": "reference", "metric": METRIC, "value": round(gbs, 4), "unit": "GB/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": describe(w), "sample": sample, "parallelism": "host cores"},
+            "cpu_baseline": {"value": round(gbs, 4), "unit": "GB/s", "cores": threads,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(gbs, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="cfg5")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--rotate", type=int, default=4)
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-tables", type=int, default=4)
+    ap.add_argument("--ref-tables", type=int, default=2)
+    ap.add_argument("--ref-budget-s", type=float, default=150.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

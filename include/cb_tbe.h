@@ -1,0 +1,164 @@
+/*
+ * cb_tbe.h -- C ABI of the GB300 pooled embedding-bag (table-batched embedding)
+ * library: the forward lookup over jagged categorical features and its
+ * de-duplicated backward.
+ *
+ * What the operation is, and where it comes from (Component Benchmark,
+ * arXiv 2609.30656):
+ *   - Abstract: recommendation models mix memory-bandwidth-bound operations
+ *     with dynamic shapes from jagged categorical features;
+ *   - Sec. I, Sec. III.B.1: the embedding tables are terabyte-scale and are
+ *     shrunk to fit one GPU;
+ *   - Sec. IV.A.2: sparse_arch performs the embedding-table lookups and is
+ *     almost entirely bandwidth-bound, with low arithmetic intensity.
+ * The paper gives no formula, so the operation is the standard pooled bag:
+ *
+ *   bag (t, b) = indices[offsets[t*B + b] .. offsets[t*B + b + 1])   (key-major)
+ *   out[b, Doff_t + j] = s_b * sum_{i in bag} w_i * E_t[indices[i], j]
+ *
+ * with Doff_t = sum of the dims of tables before t, s_b = 1 (sum pooling) or
+ * 1/L (mean pooling, L = bag length; an empty bag gives exact zeros), and
+ * w_i the per-sample weight (1 without weights). A weighted mean divides by L,
+ * not by the sum of the weights.
+ *
+ * Conventions shared by every call:
+ *   - Pointers named "device" are device memory of the current CUDA device;
+ *     the caller owns all of them (tables, indices, offsets, weights, outputs)
+ *     and keeps them alive until the work on `stream` has finished.
+ *   - All GPU work is enqueued on `stream` (0 = legacy default stream); the
+ *     calls return without waiting unless CB_VALIDATE is set.
+ *   - A handle is not thread-safe. Calls on one handle must be ordered on one
+ *     stream, or the caller synchronises between streams.
+ *   - Host-side argument errors return at once, before any GPU work.
+ *     Device-side checks (index range; offsets under CB_VALIDATE) never trap:
+ *     they set a sticky error word. Under CB_VALIDATE the call synchronises
+ *     `stream` and returns that error; otherwise cb_tbe_get_error() returns
+ *     it later. An out-of-range index contributes nothing to the output.
+ *   - Results are deterministic: the same inputs give bit-identical outputs.
+ */
+#ifndef CB_TBE_H
+#define CB_TBE_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CB_OK = 0,
+    CB_ERR_INVALID_ARG = 1, /* bad pointer, size, dtype, alignment or layout */
+    CB_ERR_INDEX_OOB = 2,   /* an index outside [0, rows_t) (device-side)    */
+    CB_ERR_BAD_OFFSETS = 3, /* offsets[0] != 0, decreasing, or last != n     */
+    CB_ERR_CAPACITY = 4,    /* sparse-gradient buffers smaller than needed   */
+    CB_ERR_OOM = 5,         /* workspace allocation failed                   */
+    CB_ERR_CUDA = 6,        /* a CUDA runtime call failed                    */
+    CB_ERR_TIMEOUT = 7      /* a bounded device-side wait gave up            */
+} cb_status;
+
+typedef enum { CB_F32 = 0, CB_F16 = 1, CB_BF16 = 2 } cb_dtype;
+typedef enum { CB_POOL_SUM = 0, CB_POOL_MEAN = 1 } cb_pooling;
+typedef enum { CB_I32 = 0, CB_I64 = 1 } cb_index_dtype;
+
+/* Flags for cb_tbe_create. */
+#define CB_VALIDATE 0x1u  /* check offsets on device; synchronise and return errors */
+#define CB_TIMING   0x2u  /* record per-component CUDA events (cb_tbe_last_timings) */
+/* Test hook: the first radix pass's tile 1 waits on a status word that nothing
+ * writes, so its bounded wait runs out and the call reports CB_ERR_TIMEOUT. */
+#define CB_DEBUG_FORCE_LOOKBACK_TIMEOUT 0x100u
+
+/* One embedding table: `rows` x `dim` values of `dtype`, row-major, at the
+ * device address `data` (16-byte aligned). dim * sizeof(dtype) must be a
+ * multiple of 16 bytes and dim at most 512. The library only reads it. */
+typedef struct {
+    const void* data;
+    int64_t rows;
+    int32_t dim;
+    cb_dtype dtype;
+} cb_table_desc;
+
+typedef struct cb_tbe cb_tbe;
+
+/* Creates a handle on the current CUDA device for `num_tables` tables (the
+ * descriptors are copied; the table memory stays the caller's). `mode` picks
+ * sum or mean pooling; `idx_dtype` is the type of both indices and offsets.
+ * The sum of all rows must be below 2^32 and num_tables * batch below 2^31.
+ * Returns CB_ERR_INVALID_ARG for a bad descriptor, CB_ERR_CUDA / CB_ERR_OOM
+ * if the device set-up fails. On success *out receives the handle. */
+cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pooling mode,
+                        cb_index_dtype idx_dtype, uint32_t flags, cb_tbe** out);
+
+/* Grows the handle's workspace for calls up to `batch` bags per table and
+ * `num_indices` lookups, so that later calls allocate nothing. Synchronises
+ * the device if it has to reallocate. */
+cb_status cb_tbe_reserve(cb_tbe* h, int32_t batch, int64_t num_indices);
+
+/* Forward (the sparse_arch lookup, Sec. IV.A.2; pooled bag defined above).
+ *   batch        B >= 0 bags per table
+ *   indices      device [num_indices], idx_dtype; row ids within each table
+ *   num_indices  n >= 0 (must equal offsets[T*B])
+ *   offsets      device [T*B + 1], idx_dtype, key-major, non-decreasing, from 0
+ *   per_sample_weights  device fp32 [n] or NULL
+ *   out          device fp32 [B, sum of dims], row-major, 16-byte aligned;
+ *                every element is written. */
+cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                         const void* offsets, const float* per_sample_weights, float* out,
+                         cudaStream_t stream);
+
+/* Row-sparse gradient written by cb_tbe_backward. All pointers are device
+ * memory owned by the caller. U = number of distinct (table, row) pairs
+ * touched by the batch; F = sum over those rows of their table's dim. */
+typedef struct {
+    int64_t* unique_ids;    /* [cap_rows] global ids row_base_t + row, ascending  */
+    int64_t* table_offsets; /* [T + 1] first entry of each table in unique_ids    */
+    int64_t* grad_offsets;  /* [cap_rows + 1] start of each row's values in grads */
+    float* grads;           /* [cap_floats] packed fp32 gradient rows; NULL = only
+                               count U and F (size query)                        */
+    int64_t cap_rows;       /* capacity of unique_ids (>= U; n always suffices)   */
+    int64_t cap_floats;     /* capacity of grads (>= F)                           */
+    int64_t* num_unique;    /* device scalar: U                                   */
+    int64_t* num_floats;    /* device scalar: F                                   */
+} cb_sparse_grad;
+
+/* Backward of the forward above with respect to the table rows, de-duplicated
+ * per touched row (the adjoint of the pooled bag; the paper profiles training
+ * steps, Sec. II and Sec. VII):
+ *   G[row_base_t + r] = sum over lookups i of table t with indices[i] == r of
+ *                       w_i * s_b(i) * grad_out[b(i), Doff_t : Doff_t + D_t]
+ * computed by an on-device stable radix sort of (row id, lookup) pairs, a
+ * run-length pass and a segmented reduction. Arguments as in cb_tbe_forward;
+ * grad_out is device fp32 [B, sum of dims], 16-byte aligned. When U > cap_rows
+ * or F > cap_floats nothing is written to unique_ids / grad_offsets / grads,
+ * num_unique and num_floats still hold the needed sizes, and the error is
+ * CB_ERR_CAPACITY (returned now under CB_VALIDATE, else by cb_tbe_get_error). */
+cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                          const void* offsets, const float* per_sample_weights,
+                          const float* grad_out, cb_sparse_grad* g, cudaStream_t stream);
+
+/* Synchronises the stream of the last call, returns the sticky device-side
+ * error (CB_OK if none) and clears it. */
+cb_status cb_tbe_get_error(cb_tbe* h);
+
+/* Per-component device times (ms) of the last call made with CB_TIMING, in the
+ * order of cb_tbe_component_name(); synchronises on the last event. Writes at
+ * most `n` entries; returns CB_ERR_INVALID_ARG without CB_TIMING. */
+cb_status cb_tbe_last_timings(cb_tbe* h, float* ms, int32_t n);
+
+/* Name of timing slot `i` ("fwd.prep", "fwd.gather", ...), NULL past the end. */
+const char* cb_tbe_component_name(int32_t i);
+
+/* Number of CUDA kernels this handle has launched since creation. */
+uint64_t cb_tbe_launch_count(const cb_tbe* h);
+
+/* Short English description of a status code. */
+const char* cb_tbe_status_string(cb_status s);
+
+/* Releases the workspace and the handle (synchronises its last stream). */
+void cb_tbe_destroy(cb_tbe* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CB_TBE_H */

@@ -1,0 +1,611 @@
+// cb_tbe.cu -- the C ABI (include/cb_tbe.h): handle, argument checks, workspace,
+// and the order of kernel launches for the forward and backward passes.
+#include <algorithm>
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "cb_tbe.h"
+#include "tbe_internal.cuh"
+#include "tbe_launch.h"
+
+using namespace cbtbe;
+
+namespace {
+
+constexpr int64_t kFwdChunk = 512;   // lookups per forward chunk
+constexpr int64_t kBwdChunk = 512;   // sorted positions per reduce chunk
+constexpr uint64_t kLookbackTimeoutNs = 1000000000ull;  // 1 s bounded wait
+constexpr int kNumTimers = 7;
+const char* const kComponentNames[kNumTimers] = {"fwd.prep",   "fwd.gather", "fwd.fixup",
+                                                 "bwd.keygen", "bwd.sort",   "bwd.rle",
+                                                 "bwd.reduce"};
+
+struct KernelClass {
+    int dtype;  // storage dtype (forward) or CB_F32 (backward)
+    int vpl;    // 16-byte vectors per lane: 1, 2 or 4
+    std::vector<int32_t> tables;
+};
+
+int elem_bytes(int dt) { return dt == CB_F32 ? 4 : 2; }
+
+int vpl_for(int row_vecs) { return row_vecs <= 32 ? 1 : (row_vecs <= 64 ? 2 : 4); }
+
+// Lanes per row and rows per warp step for a row of `vecs` 16-byte vectors.
+void lane_split(int vecs, int32_t* lanes, int32_t* groups) {
+    if (vecs >= 32) {
+        *lanes = 32;
+        *groups = 1;
+    } else if ((vecs & (vecs - 1)) == 0) {
+        *lanes = vecs;
+        *groups = 32 / vecs;
+    } else {
+        *lanes = vecs;  // not a power of two: one row per warp step
+        *groups = 1;
+    }
+}
+
+size_t align_up(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// Bump layout of the per-call workspace (pointers assigned when base != null).
+struct Workspace {
+    int64_t* table_pos = nullptr;
+    int64_t* ord_chunk_base = nullptr;
+    int64_t* class_chunk_base = nullptr;
+    Chunk* chunks = nullptr;
+    float* carry_head = nullptr;
+    float* carry_tail = nullptr;
+    int64_t* tail_owner = nullptr;
+    int64_t max_chunks = 0;
+    // backward
+    uint32_t* keys[2] = {nullptr, nullptr};
+    uint32_t* vals[2] = {nullptr, nullptr};
+    uint2* packed = nullptr;
+    uint32_t* hist = nullptr;
+    uint32_t* digit_base = nullptr;
+    uint32_t* status = nullptr;
+    uint32_t* tile_counters = nullptr;
+    int64_t* tile_heads = nullptr;
+    int64_t* tile_base = nullptr;
+    uint32_t* uniq = nullptr;
+    uint32_t* seg_start = nullptr;
+    int64_t* table_first = nullptr;
+    int64_t* float_base = nullptr;
+    int64_t* num_unique = nullptr;
+    int* cap_fail = nullptr;
+    int64_t sort_tiles = 0;
+    size_t status_bytes = 0;
+};
+
+}  // namespace
+
+struct cb_tbe {
+    int device = 0;
+    int num_sms = 1;
+    int32_t T = 0;
+    int mode = CB_POOL_SUM;
+    int is32 = 0;
+    uint32_t flags = 0;
+    int32_t sum_d = 0;
+    int32_t dmax = 0;
+    int64_t sum_rows = 0;
+    int key_bits = 1;
+    int passes = 1;
+    std::vector<TableDev> tables;
+    std::vector<KernelClass> fwd_classes, bwd_classes;
+    // persistent device memory: tables, class lists, error word, a never-written word
+    void* persist = nullptr;
+    TableDev* d_tables = nullptr;
+    int32_t* d_fwd_class_tables = nullptr;
+    int32_t* d_fwd_class_start = nullptr;
+    int32_t* d_bwd_class_tables = nullptr;
+    int32_t* d_bwd_class_start = nullptr;
+    int* d_error = nullptr;
+    uint32_t* d_never_set = nullptr;
+    // grown on demand
+    void* ws = nullptr;
+    size_t ws_bytes = 0;
+    cudaStream_t last_stream = nullptr;
+    cudaEvent_t ev_fwd[4] = {};
+    cudaEvent_t ev_bwd[5] = {};
+    bool fwd_timed = false;
+    bool bwd_timed = false;
+    uint64_t launches = 0;
+};
+
+namespace {
+
+// Computes (and, with a base, assigns) the workspace for calls up to B bags per
+// table and n lookups. Returns the byte size.
+size_t layout(const cb_tbe* h, int64_t B, int64_t n, char* base, Workspace* w) {
+    size_t off = 0;
+    auto take = [&](size_t bytes) -> void* {
+        void* p = base ? static_cast<void*>(base + off) : nullptr;
+        off += align_up(std::max<size_t>(bytes, 1));
+        return p;
+    };
+    const int64_t T = h->T;
+    const int64_t nc = std::max<size_t>(h->fwd_classes.size(), h->bwd_classes.size());
+    const int64_t chunk = std::min(kFwdChunk, kBwdChunk);
+    const int64_t max_chunks = n / chunk + T + 1;
+    Workspace ws;
+    ws.max_chunks = max_chunks;
+    ws.table_pos = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.ord_chunk_base = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.class_chunk_base = static_cast<int64_t*>(take(sizeof(int64_t) * (nc + 1)));
+    ws.chunks = static_cast<Chunk*>(take(sizeof(Chunk) * max_chunks));
+    ws.carry_head = static_cast<float*>(take(sizeof(float) * max_chunks * h->dmax));
+    ws.carry_tail = static_cast<float*>(take(sizeof(float) * max_chunks * h->dmax));
+    ws.tail_owner = static_cast<int64_t*>(take(sizeof(int64_t) * max_chunks));
+    for (int i = 0; i < 2; ++i) {
+        ws.keys[i] = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
+        ws.vals[i] = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
+    }
+    ws.packed = static_cast<uint2*>(take(sizeof(uint2) * n));
+    ws.hist = static_cast<uint32_t*>(take(sizeof(uint32_t) * 4 * 256));
+    ws.digit_base = static_cast<uint32_t*>(take(sizeof(uint32_t) * 4 * 256));
+    ws.sort_tiles = sort_num_tiles(n);
+    ws.status_bytes = sizeof(uint32_t) * static_cast<size_t>(h->passes) * ws.sort_tiles * 256;
+    // status and tile counters are adjacent so that one memset clears both
+    ws.status = static_cast<uint32_t*>(take(ws.status_bytes + sizeof(uint32_t) * 4));
+    ws.tile_counters = base ? ws.status + static_cast<size_t>(h->passes) * ws.sort_tiles * 256 : nullptr;
+    const int64_t rt = rle_num_tiles(n);
+    ws.tile_heads = static_cast<int64_t*>(take(sizeof(int64_t) * rt));
+    ws.tile_base = static_cast<int64_t*>(take(sizeof(int64_t) * rt));
+    ws.uniq = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
+    ws.seg_start = static_cast<uint32_t*>(take(sizeof(uint32_t) * (n + 1)));
+    ws.table_first = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.float_base = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.num_unique = static_cast<int64_t*>(take(sizeof(int64_t)));
+    ws.cap_fail = static_cast<int*>(take(sizeof(int)));
+    if (w) *w = ws;
+    return off;
+}
+
+cb_status ensure_workspace(cb_tbe* h, int64_t B, int64_t n) {
+    const size_t need = layout(h, B, n, nullptr, nullptr);
+    if (need <= h->ws_bytes) return CB_OK;
+    if (h->ws) {
+        cudaDeviceSynchronize();
+        cudaFree(h->ws);
+        h->ws = nullptr;
+        h->ws_bytes = 0;
+    }
+    if (cudaMalloc(&h->ws, need) != cudaSuccess) {
+        cudaGetLastError();
+        h->ws = nullptr;
+        return CB_ERR_OOM;
+    }
+    h->ws_bytes = need;
+    return CB_OK;
+}
+
+bool current_device_ok(const cb_tbe* h) {
+    int dev = -1;
+    return cudaGetDevice(&dev) == cudaSuccess && dev == h->device;
+}
+
+Problem make_problem(const cb_tbe* h, int32_t B, const void* indices, int64_t n, const void* offsets,
+                     const float* weights) {
+    Problem P;
+    P.tables = h->d_tables;
+    P.indices = indices;
+    P.offsets = offsets;
+    P.weights = weights;
+    P.error = h->d_error;
+    P.n = n;
+    P.T = h->T;
+    P.B = B;
+    P.sum_d = h->sum_d;
+    P.is32 = h->is32;
+    P.mean = h->mode == CB_POOL_MEAN;
+    P.dmax = h->dmax;
+    return P;
+}
+
+Plan make_plan(const cb_tbe* h, const Workspace& w, bool bwd, int64_t chunk_len) {
+    Plan Q;
+    Q.chunk_len = static_cast<int32_t>(chunk_len);
+    Q.num_classes = static_cast<int32_t>(bwd ? h->bwd_classes.size() : h->fwd_classes.size());
+    Q.class_tables = bwd ? h->d_bwd_class_tables : h->d_fwd_class_tables;
+    Q.class_table_start = bwd ? h->d_bwd_class_start : h->d_fwd_class_start;
+    Q.table_pos = w.table_pos;
+    Q.ord_chunk_base = w.ord_chunk_base;
+    Q.class_chunk_base = w.class_chunk_base;
+    Q.chunks = w.chunks;
+    Q.max_chunks = w.max_chunks;
+    Q.carry_head = w.carry_head;
+    Q.carry_tail = w.carry_tail;
+    Q.tail_owner = w.tail_owner;
+    return Q;
+}
+
+cb_status finish_call(cb_tbe* h, cudaStream_t stream) {
+    if (cudaGetLastError() != cudaSuccess) return CB_ERR_CUDA;
+    h->last_stream = stream;
+    if (h->flags & CB_VALIDATE) return cb_tbe_get_error(h);
+    return CB_OK;
+}
+
+void record(cb_tbe* h, cudaEvent_t e, cudaStream_t s) {
+    if (h->flags & CB_TIMING) cudaEventRecord(e, s);
+}
+
+cb_status check_common(const cb_tbe* h, int32_t batch, const void* indices, int64_t n,
+                       const void* offsets) {
+    if (!h || batch < 0 || n < 0 || !offsets || (n > 0 && !indices)) return CB_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(h->T) * batch >= (int64_t(1) << 31)) return CB_ERR_INVALID_ARG;
+    return CB_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* cb_tbe_status_string(cb_status s) {
+    switch (s) {
+        case CB_OK: return "ok";
+        case CB_ERR_INVALID_ARG: return "invalid argument";
+        case CB_ERR_INDEX_OOB: return "index out of range";
+        case CB_ERR_BAD_OFFSETS: return "malformed offsets";
+        case CB_ERR_CAPACITY: return "sparse-gradient capacity too small";
+        case CB_ERR_OOM: return "out of device memory";
+        case CB_ERR_CUDA: return "CUDA runtime error";
+        case CB_ERR_TIMEOUT: return "bounded device wait timed out";
+    }
+    return "unknown status";
+}
+
+const char* cb_tbe_component_name(int32_t i) {
+    return (i >= 0 && i < kNumTimers) ? kComponentNames[i] : nullptr;
+}
+
+cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pooling mode,
+                        cb_index_dtype idx_dtype, uint32_t flags, cb_tbe** out) {
+    if (!out || !tables || num_tables <= 0) return CB_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (mode != CB_POOL_SUM && mode != CB_POOL_MEAN) return CB_ERR_INVALID_ARG;
+    if (idx_dtype != CB_I32 && idx_dtype != CB_I64) return CB_ERR_INVALID_ARG;
+    auto* h = new (std::nothrow) cb_tbe();
+    if (!h) return CB_ERR_OOM;
+    h->T = num_tables;
+    h->mode = mode;
+    h->is32 = idx_dtype == CB_I32;
+    h->flags = flags;
+    int64_t row_base = 0, doff = 0;
+    for (int32_t t = 0; t < num_tables; ++t) {
+        const cb_table_desc& d = tables[t];
+        const bool dt_ok = d.dtype == CB_F32 || d.dtype == CB_F16 || d.dtype == CB_BF16;
+        if (!dt_ok || d.rows < 0 || d.dim <= 0 || (d.rows > 0 && !d.data) ||
+            (reinterpret_cast<uintptr_t>(d.data) & 15u)) {
+            delete h;
+            return CB_ERR_INVALID_ARG;
+        }
+        const int64_t row_bytes = static_cast<int64_t>(d.dim) * elem_bytes(d.dtype);
+        if (row_bytes % 16 != 0 || row_bytes > 2048) {
+            delete h;
+            return CB_ERR_INVALID_ARG;
+        }
+        TableDev td{};
+        td.data = d.data;
+        td.rows = d.rows;
+        td.row_base = row_base;
+        td.dim = d.dim;
+        td.doff = static_cast<int32_t>(doff);
+        td.dtype = d.dtype;
+        td.row_vecs = static_cast<int32_t>(row_bytes / 16);
+        lane_split(td.row_vecs, &td.lanes, &td.groups);
+        td.grad_vecs = d.dim / 4;
+        lane_split(td.grad_vecs, &td.grad_lanes, &td.grad_groups);
+        row_base += d.rows;
+        doff += d.dim;
+        h->dmax = std::max(h->dmax, d.dim);
+        h->tables.push_back(td);
+    }
+    if (row_base >= (int64_t(1) << 32) || doff >= (int64_t(1) << 31) || h->dmax > 512) {
+        delete h;
+        return CB_ERR_INVALID_ARG;
+    }
+    h->sum_rows = row_base;
+    h->sum_d = static_cast<int32_t>(doff);
+    int bits = 1;
+    while (bits < 32 && (int64_t(1) << bits) < row_base) ++bits;
+    h->key_bits = bits;
+    h->passes = (bits + 7) / 8;
+
+    // Kernel classes: forward by (storage dtype, vectors per lane), backward by
+    // vectors per lane of the fp32 gradient row.
+    for (int32_t t = 0; t < num_tables; ++t) {
+        TableDev& td = h->tables[t];
+        const int fv = vpl_for(td.row_vecs), bv = vpl_for(td.grad_vecs);
+        auto put = [&](std::vector<KernelClass>& cls, int dt, int v) {
+            for (size_t c = 0; c < cls.size(); ++c)
+                if (cls[c].dtype == dt && cls[c].vpl == v) {
+                    cls[c].tables.push_back(t);
+                    return static_cast<int>(c);
+                }
+            cls.push_back({dt, v, {t}});
+            return static_cast<int>(cls.size() - 1);
+        };
+        td.fwd_class = put(h->fwd_classes, td.dtype, fv);
+        td.bwd_class = put(h->bwd_classes, CB_F32, bv);
+    }
+
+    if (cudaGetDevice(&h->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device) != cudaSuccess) {
+        cudaGetLastError();
+        delete h;
+        return CB_ERR_CUDA;
+    }
+    // Persistent block: tables | fwd class tables | fwd starts | bwd class tables | bwd starts | error | never-set
+    std::vector<int32_t> fct, fcs{0}, bct, bcs{0};
+    for (auto& c : h->fwd_classes) {
+        fct.insert(fct.end(), c.tables.begin(), c.tables.end());
+        fcs.push_back(static_cast<int32_t>(fct.size()));
+    }
+    for (auto& c : h->bwd_classes) {
+        bct.insert(bct.end(), c.tables.begin(), c.tables.end());
+        bcs.push_back(static_cast<int32_t>(bct.size()));
+    }
+    size_t off = 0;
+    const size_t o_tab = off; off += align_up(sizeof(TableDev) * num_tables);
+    const size_t o_fct = off; off += align_up(sizeof(int32_t) * fct.size());
+    const size_t o_fcs = off; off += align_up(sizeof(int32_t) * fcs.size());
+    const size_t o_bct = off; off += align_up(sizeof(int32_t) * bct.size());
+    const size_t o_bcs = off; off += align_up(sizeof(int32_t) * bcs.size());
+    const size_t o_err = off; off += align_up(sizeof(int) + sizeof(uint32_t));
+    if (cudaMalloc(&h->persist, off) != cudaSuccess) {
+        cudaGetLastError();
+        delete h;
+        return CB_ERR_OOM;
+    }
+    char* p = static_cast<char*>(h->persist);
+    h->d_tables = reinterpret_cast<TableDev*>(p + o_tab);
+    h->d_fwd_class_tables = reinterpret_cast<int32_t*>(p + o_fct);
+    h->d_fwd_class_start = reinterpret_cast<int32_t*>(p + o_fcs);
+    h->d_bwd_class_tables = reinterpret_cast<int32_t*>(p + o_bct);
+    h->d_bwd_class_start = reinterpret_cast<int32_t*>(p + o_bcs);
+    h->d_error = reinterpret_cast<int*>(p + o_err);
+    h->d_never_set = reinterpret_cast<uint32_t*>(p + o_err + sizeof(int));
+    bool ok = cudaMemcpy(h->d_tables, h->tables.data(), sizeof(TableDev) * num_tables,
+                         cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemcpy(h->d_fwd_class_tables, fct.data(), sizeof(int32_t) * fct.size(),
+                          cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemcpy(h->d_fwd_class_start, fcs.data(), sizeof(int32_t) * fcs.size(),
+                          cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemcpy(h->d_bwd_class_tables, bct.data(), sizeof(int32_t) * bct.size(),
+                          cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemcpy(h->d_bwd_class_start, bcs.data(), sizeof(int32_t) * bcs.size(),
+                          cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemset(h->d_error, 0, sizeof(int) + sizeof(uint32_t)) == cudaSuccess;
+    if (ok && (flags & CB_TIMING)) {
+        for (auto& e : h->ev_fwd) ok = ok && cudaEventCreate(&e) == cudaSuccess;
+        for (auto& e : h->ev_bwd) ok = ok && cudaEventCreate(&e) == cudaSuccess;
+    }
+    if (!ok) {
+        cudaGetLastError();
+        cb_tbe_destroy(h);
+        return CB_ERR_CUDA;
+    }
+    *out = h;
+    return CB_OK;
+}
+
+cb_status cb_tbe_reserve(cb_tbe* h, int32_t batch, int64_t num_indices) {
+    if (!h || batch < 0 || num_indices < 0) return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    return ensure_workspace(h, batch, num_indices);
+}
+
+cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                         const void* offsets, const float* per_sample_weights, float* out,
+                         cudaStream_t stream) {
+    cb_status st = check_common(h, batch, indices, num_indices, offsets);
+    if (st != CB_OK) return st;
+    if (batch > 0 && (!out || (reinterpret_cast<uintptr_t>(out) & 15u))) return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    h->last_stream = stream;
+    h->fwd_timed = false;
+    if (batch == 0) return CB_OK;
+    const int64_t n = num_indices;
+    Problem P = make_problem(h, batch, indices, n, offsets, per_sample_weights);
+    record(h, h->ev_fwd[0], stream);
+    if (h->flags & CB_VALIDATE) {
+        launch_validate_offsets(P, h->num_sms, stream);
+        h->launches += 1;
+    }
+    if (n == 0) {
+        if (cudaMemsetAsync(out, 0, sizeof(float) * batch * h->sum_d, stream) != cudaSuccess)
+            return CB_ERR_CUDA;
+        return finish_call(h, stream);
+    }
+    st = ensure_workspace(h, batch, n);
+    if (st != CB_OK) return st;
+    Workspace w;
+    layout(h, batch, n, static_cast<char*>(h->ws), &w);
+    Plan Q = make_plan(h, w, false, kFwdChunk);
+    const int64_t bound = n / kFwdChunk + h->T + 1;
+    launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
+    h->launches += 2;
+    record(h, h->ev_fwd[1], stream);
+    for (size_t c = 0; c < h->fwd_classes.size(); ++c) {
+        launch_fwd_gather(P, Q, out, static_cast<int>(c), h->fwd_classes[c].dtype,
+                          h->fwd_classes[c].vpl, bound, h->num_sms, stream);
+        h->launches += 1;
+    }
+    record(h, h->ev_fwd[2], stream);
+    launch_fwd_fixup(P, Q, out, bound, h->num_sms, stream);
+    h->launches += 1;
+    record(h, h->ev_fwd[3], stream);
+    h->fwd_timed = (h->flags & CB_TIMING) != 0;
+    return finish_call(h, stream);
+}
+
+cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                          const void* offsets, const float* per_sample_weights,
+                          const float* grad_out, cb_sparse_grad* g, cudaStream_t stream) {
+    cb_status st = check_common(h, batch, indices, num_indices, offsets);
+    if (st != CB_OK) return st;
+    if (!g || !g->table_offsets || !g->num_unique || !g->num_floats) return CB_ERR_INVALID_ARG;
+    if (g->grads && (!g->unique_ids || !g->grad_offsets || g->cap_rows < 0 || g->cap_floats < 0 ||
+                     (reinterpret_cast<uintptr_t>(g->grads) & 15u)))
+        return CB_ERR_INVALID_ARG;
+    const int64_t n = num_indices;
+    if (n >= (int64_t(1) << 30)) return CB_ERR_INVALID_ARG;
+    if (n > 0 && batch > 0 && (!grad_out || (reinterpret_cast<uintptr_t>(grad_out) & 15u)))
+        return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    h->last_stream = stream;
+    h->bwd_timed = false;
+    Problem P = make_problem(h, batch, indices, n, offsets, per_sample_weights);
+    record(h, h->ev_bwd[0], stream);
+    if ((h->flags & CB_VALIDATE) && batch > 0) {
+        launch_validate_offsets(P, h->num_sms, stream);
+        h->launches += 1;
+    }
+    if (n == 0 || batch == 0) {
+        bool ok = cudaMemsetAsync(g->table_offsets, 0, sizeof(int64_t) * (h->T + 1), stream) == cudaSuccess;
+        ok = ok && cudaMemsetAsync(g->num_unique, 0, sizeof(int64_t), stream) == cudaSuccess;
+        ok = ok && cudaMemsetAsync(g->num_floats, 0, sizeof(int64_t), stream) == cudaSuccess;
+        if (g->grads) ok = ok && cudaMemsetAsync(g->grad_offsets, 0, sizeof(int64_t), stream) == cudaSuccess;
+        if (!ok) return CB_ERR_CUDA;
+        return finish_call(h, stream);
+    }
+    st = ensure_workspace(h, batch, n);
+    if (st != CB_OK) return st;
+    Workspace w;
+    layout(h, batch, n, static_cast<char*>(h->ws), &w);
+    Plan Q = make_plan(h, w, true, kBwdChunk);
+    const int64_t bound = n / kBwdChunk + h->T + 1;
+    const bool packed = per_sample_weights != nullptr || h->mode == CB_POOL_MEAN;
+
+    // (1) keys and digit histograms
+    launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
+    h->launches += 2;
+    if (cudaMemsetAsync(w.hist, 0, sizeof(uint32_t) * 4 * 256, stream) != cudaSuccess ||
+        cudaMemsetAsync(w.status, 0, w.status_bytes + sizeof(uint32_t) * 4, stream) != cudaSuccess)
+        return CB_ERR_CUDA;
+    KeyGen K;
+    K.keys = w.keys[0];
+    K.vals = w.vals[0];
+    K.packed = packed ? w.packed : nullptr;
+    K.hist = w.hist;
+    K.passes = h->passes;
+    launch_keygen(P, Q, K, packed, bound, h->num_sms, stream);
+    h->launches += 1;
+    record(h, h->ev_bwd[1], stream);
+
+    // (2) radix sort, 8 bits per pass
+    launch_digit_scan(w.hist, w.digit_base, h->passes, stream);
+    h->launches += 1;
+    int cur = 0;
+    for (int p = 0; p < h->passes; ++p) {
+        SortPass S;
+        S.keys_in = w.keys[cur];
+        S.vals_in = w.vals[cur];
+        S.keys_out = w.keys[cur ^ 1];
+        S.vals_out = w.vals[cur ^ 1];
+        S.n = n;
+        S.shift = 8 * p;
+        S.digit_base = w.digit_base + 256 * p;
+        S.status = w.status + static_cast<size_t>(p) * w.sort_tiles * 256;
+        S.tile_counter = w.tile_counters + p;
+        S.never_set = h->d_never_set;
+        S.force_timeout = (h->flags & CB_DEBUG_FORCE_LOOKBACK_TIMEOUT) && p == 0;
+        S.error = h->d_error;
+        S.timeout_ns = kLookbackTimeoutNs;
+        launch_onesweep(S, stream);
+        h->launches += 1;
+        cur ^= 1;
+    }
+    record(h, h->ev_bwd[2], stream);
+
+    // (3) runs of equal ids, (4) per-table ranges and capacity check
+    launch_rle(w.keys[cur], n, w.tile_heads, w.tile_base, w.num_unique, w.uniq, w.seg_start, stream);
+    h->launches += 3;
+    BwdOut O;
+    O.seg_start = w.seg_start;
+    O.vals_sorted = w.vals[cur];
+    O.packed = packed ? w.packed : nullptr;
+    O.uniq = w.uniq;
+    O.num_unique_ws = w.num_unique;
+    O.table_first = w.table_first;
+    O.float_base = w.float_base;
+    O.cap_fail = w.cap_fail;
+    O.unique_ids = g->unique_ids;
+    O.table_offsets = g->table_offsets;
+    O.grad_offsets = g->grad_offsets;
+    O.grads = g->grads;
+    O.cap_rows = g->cap_rows;
+    O.cap_floats = g->cap_floats;
+    O.num_unique = g->num_unique;
+    O.num_floats = g->num_floats;
+    launch_bwd_finalize(P, O, stream);
+    h->launches += 1;
+    if (g->grads) launch_plan(P, Q, 1, w.seg_start, w.num_unique, h->num_sms, false, stream);
+    if (g->grads) h->launches += 1;
+    record(h, h->ev_bwd[3], stream);
+
+    // (5) segmented reduce, (6) fix-up of runs split across chunks
+    if (g->grads) {
+        for (size_t c = 0; c < h->bwd_classes.size(); ++c) {
+            launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl, packed,
+                              bound, h->num_sms, stream);
+            h->launches += 1;
+        }
+        launch_bwd_fixup(P, Q, O, bound, h->num_sms, stream);
+        h->launches += 1;
+    }
+    record(h, h->ev_bwd[4], stream);
+    h->bwd_timed = (h->flags & CB_TIMING) != 0;
+    return finish_call(h, stream);
+}
+
+cb_status cb_tbe_get_error(cb_tbe* h) {
+    if (!h) return CB_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) {
+        cudaGetLastError();
+        return CB_ERR_CUDA;
+    }
+    int err = 0;
+    if (cudaMemcpy(&err, h->d_error, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemset(h->d_error, 0, sizeof(int)) != cudaSuccess) {
+        cudaGetLastError();
+        return CB_ERR_CUDA;
+    }
+    return static_cast<cb_status>(err);
+}
+
+cb_status cb_tbe_last_timings(cb_tbe* h, float* ms, int32_t n) {
+    if (!h || !ms || n < 0 || !(h->flags & CB_TIMING)) return CB_ERR_INVALID_ARG;
+    float v[kNumTimers];
+    for (float& x : v) x = -1.f;
+    if (h->fwd_timed) {
+        if (cudaEventSynchronize(h->ev_fwd[3]) != cudaSuccess) return CB_ERR_CUDA;
+        for (int i = 0; i < 3; ++i) cudaEventElapsedTime(&v[i], h->ev_fwd[i], h->ev_fwd[i + 1]);
+    }
+    if (h->bwd_timed) {
+        if (cudaEventSynchronize(h->ev_bwd[4]) != cudaSuccess) return CB_ERR_CUDA;
+        for (int i = 0; i < 4; ++i) cudaEventElapsedTime(&v[3 + i], h->ev_bwd[i], h->ev_bwd[i + 1]);
+    }
+    for (int i = 0; i < n && i < kNumTimers; ++i) ms[i] = v[i];
+    return CB_OK;
+}
+
+uint64_t cb_tbe_launch_count(const cb_tbe* h) { return h ? h->launches : 0; }
+
+void cb_tbe_destroy(cb_tbe* h) {
+    if (!h) return;
+    cudaStreamSynchronize(h->last_stream);
+    if (h->ws) cudaFree(h->ws);
+    if (h->persist) cudaFree(h->persist);
+    for (auto& e : h->ev_fwd)
+        if (e) cudaEventDestroy(e);
+    for (auto& e : h->ev_bwd)
+        if (e) cudaEventDestroy(e);
+    cudaGetLastError();
+    delete h;
+}
+
+}  // extern "C"

@@ -1,0 +1,436 @@
+// tbe_backward.cu -- de-duplicated backward of the pooled embedding bag with
+// respect to the table rows (the adjoint of the sparse_arch lookup, Sec. IV.A.2):
+//   G[row_base_t + r] = sum_{i : table t, indices[i] == r} w_i * s_b(i) * grad_out[b(i), Doff_t ..]
+//
+// Steps: (1) key generation: one warp per chunk of lookups walks the bags and
+// writes key_i = row_base_t + indices[i] with a payload (the bag id, or the
+// lookup position plus a packed (bag, w_i * s_b) pair when a coefficient is
+// needed), counting the radix digit histograms on the way; (2) radix sort;
+// (3) run-length pass over the sorted ids; (4) per-table unique ranges and
+// packed gradient offsets; (5) segmented reduce of the gathered grad_out
+// slices, one warp per chunk of sorted positions; (6) fp64 fix-up of runs that
+// straddle chunks.
+#include "tbe_internal.cuh"
+#include "tbe_launch.h"
+
+namespace cbtbe {
+
+constexpr int kRleThreads = 256;
+constexpr int kRleItems = 16;
+constexpr int kRleTile = kRleThreads * kRleItems;
+
+// ---------------------------------------------------------------- (1) keys
+
+template <bool PACKED>
+__global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q, KeyGen K) {
+    __shared__ uint32_t sh_hist[4 * 256];
+    for (int i = threadIdx.x; i < 4 * 256; i += blockDim.x) sh_hist[i] = 0;
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    for (int64_t j = warp_id_global(); j < total; j += warps_in_grid()) {
+        const Chunk ch = Q.chunks[j];
+        const int t = ch.table;
+        const TableDev& td = P.tables[t];
+        const int64_t k0 = ch.k0, k1 = ch.k0 + (ch.len & 0x7fffffffu);
+        const int64_t bag_lo = static_cast<int64_t>(t) * P.B, bag_hi = bag_lo + P.B;
+        // Window of 32 bag ends: lane i holds the end of bag win + i.
+        int64_t win = ch.first;
+        int64_t win_start = win < bag_hi ? load_index(P.offsets, win, P.is32) : kNoSeg;
+        int64_t my_end = (win + lane < bag_hi) ? load_index(P.offsets, win + lane + 1, P.is32) : kNoSeg;
+        for (int64_t base = k0; base < k1; base += 32) {
+            const int64_t q = base + lane;
+            const bool valid = q < k1;
+            int64_t my_bag = -1, my_s = 0, my_e = 0;
+            while (true) {
+                int cnt = 0;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) cnt += (__shfl_sync(kFull, my_end, i) <= q) ? 1 : 0;
+                const int64_t e_sel = __shfl_sync(kFull, my_end, cnt < 32 ? cnt : 31);
+                const int64_t s_sel = __shfl_sync(kFull, my_end, cnt > 0 ? cnt - 1 : 0);
+                if (valid && my_bag < 0 && cnt < 32) {
+                    my_bag = win + cnt;
+                    my_e = e_sel;
+                    my_s = cnt > 0 ? s_sel : win_start;
+                }
+                if (!__any_sync(kFull, valid && my_bag < 0)) break;
+                win_start = __shfl_sync(kFull, my_end, 31);
+                win += 32;
+                my_end = (win + lane < bag_hi) ? load_index(P.offsets, win + lane + 1, P.is32) : kNoSeg;
+            }
+            if (valid) {
+                if (my_bag >= bag_hi) {  // only reachable with malformed offsets
+                    set_error(P.error, CB_ERR_BAD_OFFSETS);
+                    my_bag = bag_hi - 1;
+                }
+                int64_t r = load_index(P.indices, q, P.is32);
+                if (r < 0 || r >= td.rows) {
+                    set_error(P.error, CB_ERR_INDEX_OOB);
+                    r = r < 0 ? 0 : td.rows - 1;
+                }
+                const uint32_t key = static_cast<uint32_t>(td.row_base + r);
+                K.keys[q] = key;
+                if (PACKED) {
+                    float c = P.weights ? __ldg(P.weights + q) : 1.f;
+                    if (P.mean && my_e > my_s) c = c / static_cast<float>(my_e - my_s);
+                    K.vals[q] = static_cast<uint32_t>(q);
+                    K.packed[q] = make_uint2(static_cast<uint32_t>(my_bag), __float_as_uint(c));
+                } else {
+                    K.vals[q] = static_cast<uint32_t>(my_bag);
+                }
+            }
+            // Digit histograms of every pass (warp-aggregated shared atomics).
+            const uint32_t vmask = __ballot_sync(kFull, valid);
+            if (valid) {
+                const uint32_t key = K.keys[q];
+                for (int p = 0; p < K.passes; ++p) {
+                    const uint32_t dgt = (key >> (8 * p)) & 255u;
+                    const uint32_t peers = __match_any_sync(vmask, dgt);
+                    if (lane == __ffs(peers) - 1) atomicAdd(&sh_hist[p * 256 + dgt], __popc(peers));
+                }
+            }
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < K.passes * 256; i += blockDim.x)
+        if (sh_hist[i]) atomicAdd(K.hist + i, sh_hist[i]);
+}
+
+// ---------------------------------------------------------------- (3) runs
+
+__device__ __forceinline__ bool is_head(const uint32_t* keys, int64_t i) {
+    return i == 0 || __ldg(keys + i) != __ldg(keys + i - 1);
+}
+
+__global__ void __launch_bounds__(kRleThreads) rle_count_kernel(const uint32_t* keys, int64_t n,
+                                                                 int64_t* tile_heads) {
+    __shared__ int64_t sh[33];
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kRleTile + threadIdx.x * kRleItems;
+    int64_t c = 0;
+    for (int i = 0; i < kRleItems; ++i)
+        if (base + i < n && is_head(keys, base + i)) ++c;
+    int64_t total;
+    block_excl_scan(c, sh, &total);
+    if (threadIdx.x == 0) tile_heads[blockIdx.x] = total;
+}
+
+__global__ void __launch_bounds__(1024) rle_scan_kernel(const int64_t* tile_heads, int64_t tiles,
+                                                        int64_t* tile_base, int64_t* num_unique) {
+    __shared__ int64_t sh[33];
+    __shared__ int64_t running;
+    if (threadIdx.x == 0) running = 0;
+    __syncthreads();
+    for (int64_t i0 = 0; i0 < tiles; i0 += blockDim.x) {
+        const int64_t i = i0 + threadIdx.x;
+        const int64_t c = i < tiles ? tile_heads[i] : 0;
+        int64_t total;
+        const int64_t ex = block_excl_scan(c, sh, &total);
+        if (i < tiles) tile_base[i] = running + ex;
+        __syncthreads();
+        if (threadIdx.x == 0) running += total;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *num_unique = running;
+}
+
+__global__ void __launch_bounds__(kRleThreads) rle_write_kernel(const uint32_t* keys, int64_t n,
+                                                                const int64_t* tile_base,
+                                                                const int64_t* num_unique,
+                                                                uint32_t* uniq, uint32_t* seg_start) {
+    __shared__ int64_t sh[33];
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kRleTile + threadIdx.x * kRleItems;
+    uint32_t flags = 0;
+    int64_t c = 0;
+    for (int i = 0; i < kRleItems; ++i)
+        if (base + i < n && is_head(keys, base + i)) {
+            flags |= 1u << i;
+            ++c;
+        }
+    int64_t total;
+    int64_t u = tile_base[blockIdx.x] + block_excl_scan(c, sh, &total);
+    for (int i = 0; i < kRleItems; ++i)
+        if (flags & (1u << i)) {
+            uniq[u] = __ldg(keys + base + i);
+            seg_start[u] = static_cast<uint32_t>(base + i);
+            ++u;
+        }
+    if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) seg_start[*num_unique] = static_cast<uint32_t>(n);
+}
+
+// ---------------------------------------------------------------- (4) ranges
+
+__global__ void __launch_bounds__(1024) bwd_finalize_kernel(Problem P, BwdOut O) {
+    __shared__ int64_t sh[33];
+    __shared__ int64_t running;
+    const int64_t U = *O.num_unique_ws;
+    for (int t = threadIdx.x; t <= P.T; t += blockDim.x) {
+        const int64_t rb = t < P.T ? P.tables[t].row_base
+                                   : P.tables[P.T - 1].row_base + P.tables[P.T - 1].rows;
+        int64_t a = 0, b = U;
+        while (a < b) {
+            const int64_t m = (a + b) >> 1;
+            if (static_cast<int64_t>(O.uniq[m]) < rb) a = m + 1; else b = m;
+        }
+        O.table_first[t] = a;
+    }
+    if (threadIdx.x == 0) running = 0;
+    __syncthreads();
+    for (int t0 = 0; t0 < P.T; t0 += blockDim.x) {
+        const int t = t0 + threadIdx.x;
+        const int64_t c = t < P.T ? (O.table_first[t + 1] - O.table_first[t]) * P.tables[t].dim : 0;
+        int64_t total;
+        const int64_t ex = block_excl_scan(c, sh, &total);
+        if (t < P.T) O.float_base[t] = running + ex;
+        __syncthreads();
+        if (threadIdx.x == 0) running += total;
+        __syncthreads();
+    }
+    const int64_t F = running;
+    for (int t = threadIdx.x; t <= P.T; t += blockDim.x) O.table_offsets[t] = O.table_first[t];
+    if (threadIdx.x == 0) {
+        O.float_base[P.T] = F;
+        *O.num_unique = U;
+        *O.num_floats = F;
+        int fail = 0;
+        // After a timed-out sort pass the sorted order is not trustworthy.
+        if (*reinterpret_cast<volatile int*>(P.error) == CB_ERR_TIMEOUT) fail = 1;
+        if (O.grads && (U > O.cap_rows || F > O.cap_floats)) {
+            set_error(P.error, CB_ERR_CAPACITY);
+            fail = 1;
+        }
+        *O.cap_fail = fail;
+        if (O.grads && !fail) O.grad_offsets[U] = F;
+    }
+}
+
+// ---------------------------------------------------------------- (5) reduce
+
+template <int VPL, bool PACKED>
+struct BwdPolicy {
+    static constexpr int kElems = 4;
+    static constexpr int kVpl = VPL;
+    static constexpr int kUnroll = 8 / VPL;
+
+    const uint32_t* seg_start;
+    const uint32_t* vals;
+    const uint2* packed;
+    const uint32_t* uniq;
+    const float* grad_out;
+    float* grads;
+    int64_t* unique_ids;
+    int64_t* grad_offsets;
+    float* carry_head;
+    float* carry_tail;
+    int64_t* tail_owner;
+    int64_t chunk;
+    int64_t n;
+    int64_t bag_lo;
+    int64_t seg_lo;      // first unique index of this table
+    int64_t float_lo;    // first float of this table in grads
+    int32_t B;
+    int32_t sum_d;
+    int32_t doff;
+    int32_t dim;
+    int32_t dmax;
+    int32_t vecs;
+
+    __device__ __forceinline__ int64_t seg_begin(int64_t s) const { return __ldg(seg_start + s); }
+    __device__ __forceinline__ int64_t seg_end(int64_t s) const { return __ldg(seg_start + s + 1); }
+    __device__ __forceinline__ void item(int64_t q, int64_t& a, float& w) const {
+        const uint32_t v = __ldg(vals + q);
+        if (PACKED) {
+            if (v >= n) {  // only after an aborted sort pass: skip the item
+                a = -1;
+                w = 0.f;
+                return;
+            }
+            const uint2 pk = __ldg(packed + v);
+            a = pk.x;
+            w = __uint_as_float(pk.y);
+        } else {
+            a = v;
+            w = 1.f;
+        }
+    }
+    __device__ __forceinline__ const uint4* row(int64_t bag, bool& ok) const {
+        const int64_t b = bag - bag_lo;
+        if (!ok || b < 0 || b >= B) {
+            ok = false;
+            return reinterpret_cast<const uint4*>(grad_out);
+        }
+        return reinterpret_cast<const uint4*>(grad_out + b * sum_d + doff);
+    }
+    __device__ __forceinline__ void unpack(const uint4& x, float (&f)[4]) const {
+        cbtbe::unpack<CB_F32>(x, f);
+    }
+    __device__ __forceinline__ void emit(int64_t seg, int64_t, int64_t, bool started, bool ends,
+                                         float (&tot)[VPL][4], int v, bool group0) const {
+        const int lane = threadIdx.x & 31;
+        if (started && lane == 0) {
+            const int64_t fo = float_lo + (seg - seg_lo) * dim;
+            unique_ids[seg] = __ldg(uniq + seg);
+            grad_offsets[seg] = fo;
+            if (!ends) tail_owner[chunk] = seg;
+        }
+        if (!group0) return;
+        float* dst;
+        if (started && ends) dst = grads + float_lo + (seg - seg_lo) * dim;
+        else dst = (started ? carry_tail : carry_head) + chunk * dmax;
+#pragma unroll
+        for (int k = 0; k < VPL; ++k) {
+            const int vec = v + 32 * k;
+            if (vec < vecs)
+                reinterpret_cast<float4*>(dst)[vec] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
+        }
+    }
+};
+
+template <int VPL, bool PACKED>
+__global__ void __launch_bounds__(kWarpThreads) bwd_reduce_kernel(Problem P, Plan Q, BwdOut O,
+                                                                  const float* grad_out, int cls) {
+    if (*O.cap_fail) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t cb = Q.class_chunk_base[cls];
+    const int64_t ce = min(Q.class_chunk_base[cls + 1], Q.max_chunks);
+    for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
+        const Chunk ch = Q.chunks[j];
+        const int t = ch.table;
+        const TableDev& td = P.tables[t];
+        BwdPolicy<VPL, PACKED> pol;
+        pol.seg_start = O.seg_start;
+        pol.vals = O.vals_sorted;
+        pol.packed = O.packed;
+        pol.uniq = O.uniq;
+        pol.grad_out = grad_out;
+        pol.grads = O.grads;
+        pol.unique_ids = O.unique_ids;
+        pol.grad_offsets = O.grad_offsets;
+        pol.carry_head = Q.carry_head;
+        pol.carry_tail = Q.carry_tail;
+        pol.tail_owner = Q.tail_owner;
+        pol.chunk = j;
+        pol.n = P.n;
+        pol.bag_lo = static_cast<int64_t>(t) * P.B;
+        pol.seg_lo = O.table_first[t];
+        pol.float_lo = O.float_base[t];
+        pol.B = P.B;
+        pol.sum_d = P.sum_d;
+        pol.doff = td.doff;
+        pol.dim = td.dim;
+        pol.dmax = P.dmax;
+        pol.vecs = td.grad_vecs;
+        ChunkCtx c;
+        c.k0 = ch.k0;
+        c.k1 = ch.k0 + (ch.len & 0x7fffffffu);
+        c.first = max(ch.first, pol.seg_lo);
+        c.seg_hi = O.table_first[t + 1];
+        c.lanes = td.grad_lanes;
+        c.groups = td.grad_groups;
+        c.row_vecs = td.grad_vecs;
+        c.last = false;
+        if (lane == 0) Q.tail_owner[j] = -1;
+        walk_chunk(pol, c, lane);
+    }
+}
+
+// ---------------------------------------------------------------- (6) fix-up
+
+__global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(Problem P, Plan Q, BwdOut O) {
+    if (*O.cap_fail) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    for (int64_t j = warp_id_global(); j < total; j += warps_in_grid()) {
+        const int64_t seg = Q.tail_owner[j];
+        if (seg < 0) continue;
+        const int t = Q.chunks[j].table;
+        const TableDev& td = P.tables[t];
+        const int64_t e = O.seg_start[seg + 1];
+        float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
+        for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
+            const float4 a = *reinterpret_cast<const float4*>(Q.carry_tail + j * P.dmax + x0);
+            double acc[4] = {a.x, a.y, a.z, a.w};
+            for (int64_t jj = j + 1; jj < total; ++jj) {
+                const Chunk c2 = Q.chunks[jj];
+                if (c2.table != t || c2.first != seg || c2.k0 >= e) break;
+                const float4 h = *reinterpret_cast<const float4*>(Q.carry_head + jj * P.dmax + x0);
+                acc[0] += h.x;
+                acc[1] += h.y;
+                acc[2] += h.z;
+                acc[3] += h.w;
+                if (e <= c2.k0 + static_cast<int64_t>(c2.len & 0x7fffffffu)) break;
+            }
+            *reinterpret_cast<float4*>(dst + x0) =
+                make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                            static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+        }
+    }
+}
+
+// ---------------------------------------------------------------- launchers
+
+template <class KernelT>
+static int occupancy_grid(KernelT kernel, int threads, int num_sms) {
+    int per_sm = 1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0) != cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    return per_sm * num_sms;
+}
+
+static int warp_grid(int64_t chunk_bound, int cap) {
+    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
+    return static_cast<int>(max64(1, min64(need, cap)));
+}
+
+void launch_keygen(const Problem& P, const Plan& Q, const KeyGen& K, bool packed, int64_t chunk_bound,
+                   int num_sms, cudaStream_t s) {
+    if (packed) {
+        static int cap = occupancy_grid(keygen_kernel<true>, kWarpThreads, num_sms);
+        keygen_kernel<true><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, K);
+    } else {
+        static int cap = occupancy_grid(keygen_kernel<false>, kWarpThreads, num_sms);
+        keygen_kernel<false><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, K);
+    }
+}
+
+int64_t rle_num_tiles(int64_t n) { return (n + kRleTile - 1) / kRleTile; }
+
+void launch_rle(const uint32_t* keys, int64_t n, int64_t* tile_heads, int64_t* tile_base,
+                int64_t* num_unique, uint32_t* uniq, uint32_t* seg_start, cudaStream_t s) {
+    const int64_t tiles = rle_num_tiles(n);
+    rle_count_kernel<<<static_cast<unsigned>(tiles), kRleThreads, 0, s>>>(keys, n, tile_heads);
+    rle_scan_kernel<<<1, 1024, 0, s>>>(tile_heads, tiles, tile_base, num_unique);
+    rle_write_kernel<<<static_cast<unsigned>(tiles), kRleThreads, 0, s>>>(keys, n, tile_base,
+                                                                         num_unique, uniq, seg_start);
+}
+
+void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s) {
+    bwd_finalize_kernel<<<1, 1024, 0, s>>>(P, O);
+}
+
+template <int VPL, bool PACKED>
+static void launch_reduce_one(const Problem& P, const Plan& Q, const BwdOut& O, const float* go,
+                              int cls, int64_t chunk_bound, int num_sms, cudaStream_t s) {
+    static int cap = occupancy_grid(bwd_reduce_kernel<VPL, PACKED>, kWarpThreads, num_sms);
+    bwd_reduce_kernel<VPL, PACKED><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, O, go, cls);
+}
+
+void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
+                       int cls, int vpl, bool packed, int64_t chunk_bound, int num_sms,
+                       cudaStream_t s) {
+#define CB_CASE(V, PK)                                                              \
+    if (vpl == V && packed == PK) {                                                 \
+        launch_reduce_one<V, PK>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s); \
+        return;                                                                     \
+    }
+    CB_CASE(1, false) CB_CASE(2, false) CB_CASE(4, false)
+    CB_CASE(1, true) CB_CASE(2, true) CB_CASE(4, true)
+#undef CB_CASE
+}
+
+void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
+                      int num_sms, cudaStream_t s) {
+    bwd_fixup_kernel<<<warp_grid(chunk_bound, num_sms * 8), kWarpThreads, 0, s>>>(P, Q, O);
+}
+
+}  // namespace cbtbe

@@ -1,0 +1,204 @@
+// tbe_forward.cu -- forward gather-pool of the pooled embedding bag
+// (sparse_arch lookups, Sec. IV.A.2; jagged categorical features, Abstract):
+//   out[b, Doff_t + j] = s_b * sum_{i in bag(t, b)} w_i * E_t[indices[i], j]
+//
+// One warp per chunk of lookup positions. A stored row is spread over V lanes
+// (16 bytes per lane per vector, V = row bytes / 16 up to 32), and a warp step
+// gathers G = 32 / V rows of the chunk at once, each lane keeping up to eight
+// 16-byte loads in flight. Rows widen to fp32 in registers; the G per-row
+// partial sums of a bag meet through warp shuffles when the bag is emitted.
+#include "tbe_internal.cuh"
+#include "tbe_launch.h"
+
+namespace cbtbe {
+
+template <int DT, int VPL>
+struct FwdPolicy {
+    static constexpr int kElems = Storage<DT>::kElems;
+    static constexpr int kVpl = VPL;
+    static constexpr int kUnroll = 8 / VPL;
+
+    const void* offsets;
+    const void* indices;
+    const float* weights;
+    const uint4* table;
+    float* out;
+    float* carry_head;
+    float* carry_tail;
+    int64_t* tail_owner;
+    int* error;
+    int64_t rows;
+    int64_t chunk;
+    int64_t bag_lo;
+    int32_t row_vecs;
+    int32_t is32;
+    int32_t sum_d;
+    int32_t doff;
+    int32_t dmax;
+    int32_t mean;
+
+    __device__ __forceinline__ int64_t seg_begin(int64_t s) const { return load_index(offsets, s, is32); }
+    __device__ __forceinline__ int64_t seg_end(int64_t s) const { return load_index(offsets, s + 1, is32); }
+    __device__ __forceinline__ void item(int64_t q, int64_t& a, float& w) const {
+        a = load_index(indices, q, is32);
+        w = weights ? __ldg(weights + q) : 1.f;
+    }
+    __device__ __forceinline__ const uint4* row(int64_t r, bool& ok) const {
+        if (!ok) return table;
+        if (r < 0 || r >= rows) {
+            set_error(error, CB_ERR_INDEX_OOB);  // contributes nothing
+            ok = false;
+            return table;
+        }
+        return table + r * row_vecs;
+    }
+    __device__ __forceinline__ void unpack(const uint4& x, float (&f)[kElems]) const {
+        cbtbe::unpack<DT>(x, f);
+    }
+    __device__ __forceinline__ void emit(int64_t bag, int64_t s, int64_t e, bool started, bool ends,
+                                         float (&tot)[VPL][kElems], int v, bool group0) const {
+        if (started && !ends && (threadIdx.x & 31) == 0) tail_owner[chunk] = bag;
+        if (!group0) return;
+        float* dst;
+        float L = 0.f;
+        if (started && ends) {
+            dst = out + (bag - bag_lo) * sum_d + doff;
+            if (mean && e > s) L = static_cast<float>(e - s);
+        } else {
+            dst = (started ? carry_tail : carry_head) + chunk * dmax;
+        }
+#pragma unroll
+        for (int k = 0; k < VPL; ++k) {
+            const int vec = v + 32 * k;
+            if (vec >= row_vecs) continue;
+            float o[kElems];
+#pragma unroll
+            for (int x = 0; x < kElems; ++x) o[x] = L > 0.f ? tot[k][x] / L : tot[k][x];
+            float4* d4 = reinterpret_cast<float4*>(dst + vec * kElems);
+#pragma unroll
+            for (int x = 0; x < kElems / 4; ++x)
+                d4[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+        }
+    }
+};
+
+template <int DT, int VPL>
+__global__ void __launch_bounds__(kWarpThreads) fwd_gather_kernel(Problem P, Plan Q, float* out,
+                                                                  int cls) {
+    const int lane = threadIdx.x & 31;
+    const int64_t cb = Q.class_chunk_base[cls];
+    const int64_t ce = min(Q.class_chunk_base[cls + 1], Q.max_chunks);
+    for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
+        const Chunk ch = Q.chunks[j];
+        const TableDev& td = P.tables[ch.table];
+        FwdPolicy<DT, VPL> pol;
+        pol.offsets = P.offsets;
+        pol.indices = P.indices;
+        pol.weights = P.weights;
+        pol.table = static_cast<const uint4*>(td.data);
+        pol.out = out;
+        pol.carry_head = Q.carry_head;
+        pol.carry_tail = Q.carry_tail;
+        pol.tail_owner = Q.tail_owner;
+        pol.error = P.error;
+        pol.rows = td.rows;
+        pol.chunk = j;
+        pol.bag_lo = static_cast<int64_t>(ch.table) * P.B;
+        pol.row_vecs = td.row_vecs;
+        pol.is32 = P.is32;
+        pol.sum_d = P.sum_d;
+        pol.doff = td.doff;
+        pol.dmax = P.dmax;
+        pol.mean = P.mean;
+        ChunkCtx c;
+        c.k0 = ch.k0;
+        c.k1 = ch.k0 + (ch.len & 0x7fffffffu);
+        c.first = ch.first;
+        c.seg_hi = pol.bag_lo + P.B;
+        c.lanes = td.lanes;
+        c.groups = td.groups;
+        c.row_vecs = td.row_vecs;
+        c.last = (ch.len >> 31) != 0;
+        if (lane == 0) Q.tail_owner[j] = -1;
+        walk_chunk(pol, c, lane);
+    }
+}
+
+// A bag split over chunks: its tail piece (chunk where it starts) plus the head
+// pieces of the following chunks, added in chunk order in fp64, then scaled.
+__global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(Problem P, Plan Q, float* out) {
+    const int lane = threadIdx.x & 31;
+    const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    for (int64_t j = warp_id_global(); j < total; j += warps_in_grid()) {
+        const int64_t bag = Q.tail_owner[j];
+        if (bag < 0) continue;
+        const int t = Q.chunks[j].table;
+        const TableDev& td = P.tables[t];
+        const int64_t s = load_index(P.offsets, bag, P.is32);
+        const int64_t e = load_index(P.offsets, bag + 1, P.is32);
+        float* dst = out + (bag - static_cast<int64_t>(t) * P.B) * P.sum_d + td.doff;
+        for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
+            const float4 a = *reinterpret_cast<const float4*>(Q.carry_tail + j * P.dmax + x0);
+            double acc[4] = {a.x, a.y, a.z, a.w};
+            for (int64_t jj = j + 1; jj < total; ++jj) {
+                const Chunk c2 = Q.chunks[jj];
+                if (c2.table != t || c2.first != bag || c2.k0 >= e) break;
+                const float4 h = *reinterpret_cast<const float4*>(Q.carry_head + jj * P.dmax + x0);
+                acc[0] += h.x;
+                acc[1] += h.y;
+                acc[2] += h.z;
+                acc[3] += h.w;
+                if (e <= c2.k0 + static_cast<int64_t>(c2.len & 0x7fffffffu)) break;
+            }
+            if (P.mean && e > s) {
+                const double L = static_cast<double>(e - s);
+                for (int x = 0; x < 4; ++x) acc[x] /= L;
+            }
+            *reinterpret_cast<float4*>(dst + x0) =
+                make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                            static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+        }
+    }
+}
+
+template <int DT, int VPL>
+static int gather_grid(int num_sms) {
+    static int per_sm = -1;
+    if (per_sm < 0) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fwd_gather_kernel<DT, VPL>,
+                                                          kWarpThreads, 0) != cudaSuccess ||
+            per_sm < 1)
+            per_sm = 1;
+    }
+    return per_sm * num_sms;
+}
+
+template <int DT, int VPL>
+static void launch_one(const Problem& P, const Plan& Q, float* out, int cls, int64_t chunk_bound,
+                       int num_sms, cudaStream_t s) {
+    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
+    const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL>(num_sms)));
+    fwd_gather_kernel<DT, VPL><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
+}
+
+void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,
+                       int64_t chunk_bound, int num_sms, cudaStream_t s) {
+#define CB_CASE(D, V)                                              \
+    if (dtype == D && vpl == V) {                                  \
+        launch_one<D, V>(P, Q, out, cls, chunk_bound, num_sms, s); \
+        return;                                                    \
+    }
+    CB_CASE(CB_F32, 1) CB_CASE(CB_F32, 2) CB_CASE(CB_F32, 4)
+    CB_CASE(CB_F16, 1) CB_CASE(CB_F16, 2) CB_CASE(CB_F16, 4)
+    CB_CASE(CB_BF16, 1) CB_CASE(CB_BF16, 2) CB_CASE(CB_BF16, 4)
+#undef CB_CASE
+}
+
+void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
+                      int num_sms, cudaStream_t s) {
+    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
+    const int grid = static_cast<int>(min64(need, static_cast<int64_t>(num_sms) * 8));
+    fwd_fixup_kernel<<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out);
+}
+
+}  // namespace cbtbe

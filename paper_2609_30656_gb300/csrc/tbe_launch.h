@@ -1,0 +1,83 @@
+// tbe_launch.h -- host-callable launchers of the kernels (internal to the library).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace cbtbe {
+
+struct Problem;
+struct Plan;
+
+// One radix pass over n (key, payload) pairs.
+struct SortPass {
+    const uint32_t* keys_in;
+    const uint32_t* vals_in;
+    uint32_t* keys_out;
+    uint32_t* vals_out;
+    int64_t n;
+    int shift;                   // digit = (key >> shift) & 255
+    const uint32_t* digit_base;  // [256] first output slot of each digit
+    uint32_t* status;            // [tiles * 256], zeroed before the pass
+    uint32_t* tile_counter;      // zeroed before the pass
+    const uint32_t* never_set;   // a zero word no kernel writes (timeout test hook)
+    int force_timeout;
+    int* error;
+    uint64_t timeout_ns;
+};
+
+struct KeyGen {
+    uint32_t* keys;    // [n] row_base_t + index
+    uint32_t* vals;    // [n] bag id, or lookup position when `packed` is used
+    uint2* packed;     // [n] (bag id, bits of w_i * s_b) by lookup position, or null
+    uint32_t* hist;    // [passes * 256], zeroed before
+    int passes;
+};
+
+struct BwdOut {
+    // workspace
+    const uint32_t* seg_start;   // [U + 1]
+    const uint32_t* vals_sorted; // [n]
+    const uint2* packed;         // [n] or null
+    const uint32_t* uniq;        // [U]
+    int64_t* num_unique_ws;
+    int64_t* table_first;        // [T + 1]
+    int64_t* float_base;         // [T + 1]
+    int* cap_fail;
+    // caller's buffers
+    int64_t* unique_ids;
+    int64_t* table_offsets;
+    int64_t* grad_offsets;
+    float* grads;
+    int64_t cap_rows;
+    int64_t cap_floats;
+    int64_t* num_unique;
+    int64_t* num_floats;
+};
+
+void launch_validate_offsets(const Problem& P, int num_sms, cudaStream_t s);
+void launch_plan(const Problem& P, const Plan& Q, int mode, const uint32_t* seg_start,
+                 const int64_t* num_unique, int num_sms, bool tables_too, cudaStream_t s);
+
+void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,
+                       int64_t chunk_bound, int num_sms, cudaStream_t s);
+void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
+                      int num_sms, cudaStream_t s);
+
+int64_t sort_num_tiles(int64_t n);
+void launch_digit_scan(const uint32_t* hist, uint32_t* base, int passes, cudaStream_t s);
+void launch_onesweep(const SortPass& S, cudaStream_t s);
+
+void launch_keygen(const Problem& P, const Plan& Q, const KeyGen& K, bool packed, int64_t chunk_bound,
+                   int num_sms, cudaStream_t s);
+int64_t rle_num_tiles(int64_t n);
+void launch_rle(const uint32_t* keys, int64_t n, int64_t* tile_heads, int64_t* tile_base,
+                int64_t* num_unique, uint32_t* uniq, uint32_t* seg_start, cudaStream_t s);
+void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s);
+void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
+                       int cls, int vpl, bool packed, int64_t chunk_bound, int num_sms,
+                       cudaStream_t s);
+void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
+                      int num_sms, cudaStream_t s);
+
+}  // namespace cbtbe

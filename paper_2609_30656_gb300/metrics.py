@@ -1,0 +1,111 @@
+"""Algorithmic byte counts of the pooled embedding bag and its backward.
+
+"Algorithmic" bytes are what the method itself must move, with every lookup's
+row counted once and nothing added for the implementation's own scratch
+traffic: the embedding module's estimated bandwidth column of the paper's
+result table (Sec. IV.A.1) divided by the achieved time gives the same
+"bandwidth utilisation" figure. Per unit:
+
+  forward   per lookup: D_t * e_S (stored row) + idx_bytes (+ 4 for a weight)
+            per bag:    idx_bytes (offsets)    per output row: sum D * 4
+  backward  per lookup: D_t * 4 (gathered grad_out slice) + idx_bytes (+ 4)
+            per bag:    idx_bytes              per unique row: 8 (id) + D_t * 4
+  sort      per lookup and pass: 16 (read and write a 4-byte key and payload)
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+
+@dataclass
+class BatchCounts:
+    """Host-side sizes of one batch; lookups_per_table from the table boundaries."""
+    num_tables: int
+    batch: int
+    dims: tuple[int, ...]
+    elem_bytes: int
+    idx_bytes: int
+    weighted: bool
+    lookups_per_table: tuple[int, ...]
+
+    @property
+    def n(self) -> int:
+        return int(sum(self.lookups_per_table))
+
+    @property
+    def sum_dims(self) -> int:
+        return int(sum(self.dims))
+
+
+def batch_counts(dims, elem_bytes: int, batch: int, offsets: torch.Tensor, weighted: bool,
+                 idx_bytes: int = 8) -> BatchCounts:
+    T = len(dims)
+    starts = offsets[::batch][:T + 1].to("cpu").tolist() if batch > 0 else [0] * (T + 1)
+    per = tuple(int(starts[t + 1] - starts[t]) for t in range(T))
+    return BatchCounts(T, batch, tuple(int(d) for d in dims), elem_bytes, idx_bytes, weighted, per)
+
+
+def forward_bytes(c: BatchCounts) -> dict[str, int]:
+    rows = sum(L * d * c.elem_bytes for L, d in zip(c.lookups_per_table, c.dims))
+    parts = {
+        "rows": rows,
+        "indices": c.n * c.idx_bytes,
+        "offsets": (c.num_tables * c.batch + 1) * c.idx_bytes,
+        "weights": c.n * 4 if c.weighted else 0,
+        "output": c.batch * c.sum_dims * 4,
+    }
+    parts["total"] = sum(parts.values())
+    return parts
+
+
+def forward_unique_bytes(c: BatchCounts, unique_per_table) -> int:
+    """Compulsory forward traffic: each distinct row read once (L2-perfect reuse)."""
+    f = forward_bytes(c)
+    rows = sum(int(u) * d * c.elem_bytes for u, d in zip(unique_per_table, c.dims))
+    return f["total"] - f["rows"] + rows
+
+
+def backward_bytes(c: BatchCounts, unique_per_table) -> dict[str, int]:
+    U = int(sum(int(u) for u in unique_per_table))
+    parts = {
+        "grad_gather": sum(L * d * 4 for L, d in zip(c.lookups_per_table, c.dims)),
+        "indices": c.n * c.idx_bytes,
+        "offsets": (c.num_tables * c.batch + 1) * c.idx_bytes,
+        "weights": c.n * 4 if c.weighted else 0,
+        "unique_ids": U * 8,
+        "grads": sum(int(u) * d * 4 for u, d in zip(unique_per_table, c.dims)),
+    }
+    parts["total"] = sum(parts.values())
+    return parts
+
+
+def sort_bytes(n: int, passes: int) -> int:
+    return 16 * n * passes
+
+
+def radix_passes(rows) -> int:
+    total = int(sum(rows))
+    bits = 1
+    while bits < 32 and (1 << bits) < total:
+        bits += 1
+    return (bits + 7) // 8
+
+
+def component_bytes(c: BatchCounts, unique_per_table, rows, packed: bool) -> dict[str, int]:
+    """Algorithmic bytes of each timed component (the kernels inside it)."""
+    f = forward_bytes(c)
+    b = backward_bytes(c, unique_per_table)
+    U = int(sum(int(u) for u in unique_per_table))
+    n = c.n
+    return {
+        "fwd.gather": f["total"],
+        "bwd.keygen": n * c.idx_bytes + (c.num_tables * c.batch + 1) * c.idx_bytes + 8 * n
+        + (12 * n if packed else 0),
+        "bwd.sort": sort_bytes(n, radix_passes(rows)),
+        "bwd.rle": 8 * n + 8 * U,
+        "bwd.reduce": b["grad_gather"] + 4 * n + (8 * n if packed else 0) + 4 * U + b["grads"]
+        + 16 * U,
+    }

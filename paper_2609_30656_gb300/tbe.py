@@ -1,0 +1,269 @@
+"""Python binding of the C ABI in include/cb_tbe.h (ctypes; argument marshalling only).
+
+Every step of the lookup and its backward runs in the CUDA kernels of
+libcb_tbe.so. PyTorch supplies device memory and the current stream. Host
+(CPU) tensors passed to ``forward`` / ``backward`` are copied to the device on
+the current stream first, which is how an end-to-end caller feeds a batch from
+pinned host memory.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libcb_tbe.so")
+
+CB_OK, CB_ERR_INVALID_ARG, CB_ERR_INDEX_OOB, CB_ERR_BAD_OFFSETS = 0, 1, 2, 3
+CB_ERR_CAPACITY, CB_ERR_OOM, CB_ERR_CUDA, CB_ERR_TIMEOUT = 4, 5, 6, 7
+CB_VALIDATE, CB_TIMING, CB_DEBUG_FORCE_LOOKBACK_TIMEOUT = 0x1, 0x2, 0x100
+_DTYPES = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2}
+_POOL = {"sum": 0, "mean": 1}
+_IDX = {torch.int32: 0, torch.int64: 1}
+
+# Every entry point declared in include/cb_tbe.h.
+EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
+           "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
+           "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy")
+
+
+class CbTableDesc(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("rows", ctypes.c_int64), ("dim", ctypes.c_int32),
+                ("dtype", ctypes.c_int)]
+
+
+class CbSparseGrad(ctypes.Structure):
+    _fields_ = [("unique_ids", ctypes.c_void_p), ("table_offsets", ctypes.c_void_p),
+                ("grad_offsets", ctypes.c_void_p), ("grads", ctypes.c_void_p),
+                ("cap_rows", ctypes.c_int64), ("cap_floats", ctypes.c_int64),
+                ("num_unique", ctypes.c_void_p), ("num_floats", ctypes.c_void_p)]
+
+
+class CbTbeError(RuntimeError):
+    def __init__(self, status: int, what: str = ""):
+        msg = _lib_status_string(status)
+        super().__init__(f"{what}: {msg} (status {status})" if what else f"{msg} (status {status})")
+        self.status = status
+
+
+_lib = None
+
+
+def load_library() -> ctypes.CDLL:
+    """Loads libcb_tbe.so; fails loudly when it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"CUDA library {LIB_PATH} is missing; build it with "
+                           "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(LIB_PATH)
+    p, i32, i64, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+    lib.cb_tbe_create.argtypes = [p, i32, ctypes.c_int, ctypes.c_int, u32, ctypes.POINTER(p)]
+    lib.cb_tbe_reserve.argtypes = [p, i32, i64]
+    lib.cb_tbe_forward.argtypes = [p, i32, p, i64, p, p, p, p]
+    lib.cb_tbe_backward.argtypes = [p, i32, p, i64, p, p, p, ctypes.POINTER(CbSparseGrad), p]
+    lib.cb_tbe_get_error.argtypes = [p]
+    lib.cb_tbe_last_timings.argtypes = [p, ctypes.POINTER(ctypes.c_float), i32]
+    lib.cb_tbe_component_name.argtypes = [i32]
+    lib.cb_tbe_component_name.restype = ctypes.c_char_p
+    lib.cb_tbe_launch_count.argtypes = [p]
+    lib.cb_tbe_launch_count.restype = ctypes.c_uint64
+    lib.cb_tbe_status_string.argtypes = [ctypes.c_int]
+    lib.cb_tbe_status_string.restype = ctypes.c_char_p
+    lib.cb_tbe_destroy.argtypes = [p]
+    lib.cb_tbe_destroy.restype = None
+    for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
+                 "cb_tbe_get_error", "cb_tbe_last_timings"):
+        getattr(lib, name).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _lib_status_string(status: int) -> str:
+    try:
+        return load_library().cb_tbe_status_string(status).decode()
+    except Exception:  # pragma: no cover - library missing
+        return f"status {status}"
+
+
+def component_names() -> list[str]:
+    lib = load_library()
+    names, i = [], 0
+    while True:
+        s = lib.cb_tbe_component_name(i)
+        if s is None:
+            return names
+        names.append(s.decode())
+        i += 1
+
+
+def _check(status: int, what: str):
+    if status != CB_OK:
+        raise CbTbeError(status, what)
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+@dataclass
+class SparseGrad:
+    """Row-sparse gradient: rows `unique_ids[:U]` with values `grads[:F]`."""
+    unique_ids: torch.Tensor     # int64 [cap_rows]
+    table_offsets: torch.Tensor  # int64 [T + 1]
+    grad_offsets: torch.Tensor   # int64 [cap_rows + 1]
+    grads: torch.Tensor | None   # fp32 [cap_floats]
+    num_unique_dev: torch.Tensor  # int64 [1]
+    num_floats_dev: torch.Tensor  # int64 [1]
+
+    @property
+    def num_unique(self) -> int:
+        return int(self.num_unique_dev.item())
+
+    @property
+    def num_floats(self) -> int:
+        return int(self.num_floats_dev.item())
+
+
+class TBE:
+    """Table-batched pooled embedding bag over caller-owned device tables."""
+
+    def __init__(self, tables: list[torch.Tensor], pooling: str = "sum",
+                 index_dtype: torch.dtype = torch.int64, validate: bool = False,
+                 timing: bool = False, extra_flags: int = 0):
+        lib = load_library()
+        if not tables:
+            raise ValueError("at least one table is needed")
+        self.device = tables[0].device
+        if self.device.type != "cuda":
+            raise ValueError("tables must be CUDA tensors")
+        for t in tables:
+            if t.device != self.device or t.dim() != 2 or not t.is_contiguous():
+                raise ValueError("tables must be contiguous 2-D tensors on one CUDA device")
+            if t.dtype not in _DTYPES:
+                raise ValueError(f"unsupported table dtype {t.dtype}")
+        self.tables = list(tables)  # the ABI borrows the memory: keep it alive
+        self.dims = [int(t.shape[1]) for t in tables]
+        self.rows = [int(t.shape[0]) for t in tables]
+        self.sum_dims = sum(self.dims)
+        self.pooling = pooling
+        self.index_dtype = index_dtype
+        descs = (CbTableDesc * len(tables))(*[
+            CbTableDesc(t.data_ptr(), int(t.shape[0]), int(t.shape[1]), _DTYPES[t.dtype])
+            for t in tables])
+        flags = (CB_VALIDATE if validate else 0) | (CB_TIMING if timing else 0) | extra_flags
+        handle = ctypes.c_void_p()
+        with torch.cuda.device(self.device):
+            _check(lib.cb_tbe_create(descs, len(tables), _POOL[pooling], _IDX[index_dtype], flags,
+                                     ctypes.byref(handle)), "cb_tbe_create")
+        self._h = handle
+        self._lib = lib
+
+    # ------------------------------------------------------------------ helpers
+    def _stream(self):
+        return ctypes.c_void_p(torch.cuda.current_stream(self.device).cuda_stream)
+
+    def _dev(self, t: torch.Tensor | None, dtype: torch.dtype | None = None):
+        if t is None:
+            return None
+        if dtype is not None and t.dtype != dtype:
+            raise TypeError(f"expected {dtype}, got {t.dtype}")
+        if t.device != self.device:
+            t = t.to(self.device, non_blocking=True)
+        return t.contiguous()
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.cb_tbe_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # ------------------------------------------------------------------ API
+    def reserve(self, batch: int, num_indices: int):
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_reserve(self._h, batch, num_indices), "cb_tbe_reserve")
+
+    def forward(self, indices: torch.Tensor, offsets: torch.Tensor,
+                per_sample_weights: torch.Tensor | None = None,
+                out: torch.Tensor | None = None) -> torch.Tensor:
+        T = len(self.dims)
+        batch = (offsets.numel() - 1) // T
+        ind = self._dev(indices, self.index_dtype)
+        off = self._dev(offsets, self.index_dtype)
+        w = self._dev(per_sample_weights, torch.float32)
+        if out is None:
+            out = torch.empty(batch, self.sum_dims, dtype=torch.float32, device=self.device)
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_forward(self._h, batch, _ptr(ind), ind.numel(), _ptr(off),
+                                            _ptr(w), _ptr(out), self._stream()), "cb_tbe_forward")
+        return out
+
+    def alloc_grad(self, cap_rows: int, cap_floats: int, size_only: bool = False) -> SparseGrad:
+        dev = self.device
+        T = len(self.dims)
+        return SparseGrad(
+            unique_ids=torch.empty(max(cap_rows, 1), dtype=torch.int64, device=dev),
+            table_offsets=torch.empty(T + 1, dtype=torch.int64, device=dev),
+            grad_offsets=torch.empty(max(cap_rows, 0) + 1, dtype=torch.int64, device=dev),
+            grads=None if size_only else torch.empty(max(cap_floats, 4), dtype=torch.float32,
+                                                     device=dev),
+            num_unique_dev=torch.zeros(1, dtype=torch.int64, device=dev),
+            num_floats_dev=torch.zeros(1, dtype=torch.int64, device=dev))
+
+    def backward_into(self, g: SparseGrad, indices, offsets, grad_out,
+                      per_sample_weights=None, cap_rows: int | None = None,
+                      cap_floats: int | None = None) -> SparseGrad:
+        T = len(self.dims)
+        batch = (offsets.numel() - 1) // T
+        ind = self._dev(indices, self.index_dtype)
+        off = self._dev(offsets, self.index_dtype)
+        w = self._dev(per_sample_weights, torch.float32)
+        go = self._dev(grad_out, torch.float32)
+        cs = CbSparseGrad(
+            g.unique_ids.data_ptr(), g.table_offsets.data_ptr(), g.grad_offsets.data_ptr(),
+            None if g.grads is None else g.grads.data_ptr(),
+            g.unique_ids.numel() if cap_rows is None else cap_rows,
+            0 if g.grads is None else (g.grads.numel() if cap_floats is None else cap_floats),
+            g.num_unique_dev.data_ptr(), g.num_floats_dev.data_ptr())
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_backward(self._h, batch, _ptr(ind), ind.numel(), _ptr(off),
+                                             _ptr(w), _ptr(go), ctypes.byref(cs), self._stream()),
+                   "cb_tbe_backward")
+        return g
+
+    def backward(self, indices, offsets, grad_out, per_sample_weights=None) -> SparseGrad:
+        """Sizes the output with a counting call, then computes the gradient."""
+        probe = self.alloc_grad(0, 0, size_only=True)
+        self.backward_into(probe, indices, offsets, grad_out, per_sample_weights)
+        U, F = probe.num_unique, probe.num_floats
+        g = self.alloc_grad(U, F)
+        return self.backward_into(g, indices, offsets, grad_out, per_sample_weights)
+
+    def get_error(self) -> int:
+        with torch.cuda.device(self.device):
+            return self._lib.cb_tbe_get_error(self._h)
+
+    def raise_on_error(self):
+        st = self.get_error()
+        if st != CB_OK:
+            raise CbTbeError(st, "device-side check")
+
+    def last_timings(self) -> dict[str, float]:
+        names = component_names()
+        buf = (ctypes.c_float * len(names))()
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_last_timings(self._h, buf, len(names)), "cb_tbe_last_timings")
+        return {n: float(v) for n, v in zip(names, buf)}
+
+    def launch_count(self) -> int:
+        return int(self._lib.cb_tbe_launch_count(self._h))

@@ -206,10 +206,13 @@ class Batch:
         return int(self.indices.numel())
 
 
-def make_tables(w: Workload, seed: int, device, int_valued: bool = False) -> list[torch.Tensor]:
-    """Row-major [rows_t, D_t] tables in the workload's storage type."""
+def make_tables(w: Workload, seed: int, device, int_valued: bool = False,
+                only=None) -> list[torch.Tensor]:
+    """Row-major [rows_t, D_t] tables in the workload's storage type (`only`: a subset)."""
     out = []
     for t, (r, d) in enumerate(zip(w.rows, w.dims)):
+        if only is not None and t not in only:
+            continue
         g = _gen(device, seed, _CFG_IDS.get(w.name.split("-")[0], 0), t, 0x7AB)
         if int_valued:
             x = torch.randint(-8, 9, (r, d), generator=g, device=torch.device(device),

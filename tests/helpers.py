@@ -91,3 +91,99 @@ def table_meta(tables):
 
 __all__ = ["random_problem", "torch_forward_f64", "torch_dense_grad_f64", "sparse_to_dense",
            "table_meta", "wl"]
+
+
+# ----------------------------------------------------------------------------- GPU parity
+
+RTOL = {torch.float32: 1e-5, torch.float16: 2e-3, torch.bfloat16: 2e-3}
+RTOL_BWD = 1e-5  # gradients are accumulated and stored in fp32 whatever the table dtype
+
+
+def forward_reference(tables_cpu, batch, indices, offsets, weights, mean):
+    """Oracle output and its condition scale S = s_b * sum_i |w_i * E[idx_i, j]|."""
+    import oracle
+    ref = oracle.forward(tables_cpu, batch, indices, offsets, weights=weights, mean=mean)
+    absw = None if weights is None else weights.abs()
+    scale = oracle.forward([t.abs() for t in tables_cpu], batch, indices, offsets, weights=absw,
+                           mean=mean)
+    return ref, scale
+
+
+def assert_forward_close(y_gpu, ref, scale, rtol, what=""):
+    y = y_gpu.detach().cpu().double().numpy()
+    assert y.shape == ref.shape
+    err = np.abs(y - ref)
+    bad = err > rtol * scale + 1e-30
+    if bad.any():
+        i = np.argwhere(bad)[0]
+        raise AssertionError(f"{what}: {int(bad.sum())} elements off; first at {tuple(i)}: "
+                             f"gpu {y[tuple(i)]!r} oracle {ref[tuple(i)]!r} scale {scale[tuple(i)]!r}")
+
+
+def backward_reference(rows, dims, batch, indices, offsets, grad_out, weights, mean):
+    import oracle
+    res = oracle.backward(rows, dims, batch, indices, offsets, grad_out, weights=weights, mean=mean)
+    absw = None if weights is None else weights.abs()
+    sc = oracle.backward(rows, dims, batch, indices, offsets, grad_out.abs(), weights=absw,
+                         mean=mean)
+    return res, sc.grads
+
+
+def assert_backward_matches(g, res, scale, rtol=RTOL_BWD, what=""):
+    U = g.num_unique
+    assert U == res.num_unique, f"{what}: U {U} vs oracle {res.num_unique}"
+    F = g.num_floats
+    assert F == int(res.grad_offsets[-1])
+    np.testing.assert_array_equal(g.unique_ids[:U].cpu().numpy(), res.uniq)
+    np.testing.assert_array_equal(g.table_offsets.cpu().numpy(), res.table_offsets)
+    np.testing.assert_array_equal(g.grad_offsets[:U + 1].cpu().numpy(), res.grad_offsets)
+    got = g.grads[:F].detach().cpu().double().numpy()
+    err = np.abs(got - res.grads)
+    bad = err > rtol * scale + 1e-30
+    if bad.any():
+        i = int(np.argwhere(bad)[0][0])
+        raise AssertionError(f"{what}: {int(bad.sum())} gradient values off; first at {i}: "
+                             f"gpu {got[i]!r} oracle {res.grads[i]!r} scale {scale[i]!r}")
+
+
+def sub_batch(indices, offsets, weights, num_tables, batch, cols):
+    """The bags (t, b) for b in `cols` of every table, as a smaller key-major batch."""
+    cols = torch.as_tensor(cols, dtype=torch.int64)
+    off = offsets.cpu()
+    ind = indices.cpu()
+    w = None if weights is None else weights.cpu()
+    new_ind, new_w, lens = [], [], []
+    for t in range(num_tables):
+        for b in cols.tolist():
+            s, e = int(off[t * batch + b]), int(off[t * batch + b + 1])
+            new_ind.append(ind[s:e])
+            if w is not None:
+                new_w.append(w[s:e])
+            lens.append(e - s)
+    o = torch.zeros(len(lens) + 1, dtype=torch.int64)
+    o[1:] = torch.cumsum(torch.tensor(lens, dtype=torch.int64), 0)
+    ii = torch.cat(new_ind) if new_ind else torch.zeros(0, dtype=ind.dtype)
+    ww = (torch.cat(new_w) if new_w else torch.zeros(0)) if w is not None else None
+    return ii.to(ind.dtype), o.to(ind.dtype), ww
+
+
+def compact_tables(tables, indices, offsets, num_tables, batch):
+    """Host copies of only the rows a batch touches, with indices renumbered.
+
+    Returns (host tables, renumbered host indices). The renumbering is a plain
+    torch.unique / searchsorted per table, so the oracle sees the same stored
+    rows at new positions: a pooled sum does not depend on where a row lives.
+    """
+    off = offsets.cpu()
+    new_tabs, new_ind = [], []
+    for t in range(num_tables):
+        s, e = int(off[t * batch]), int(off[(t + 1) * batch])
+        idx = indices[s:e]
+        if idx.numel() == 0:
+            new_tabs.append(tables[t][:1].cpu())
+            new_ind.append(idx.cpu())
+            continue
+        uniq = torch.unique(idx)
+        new_tabs.append(tables[t].index_select(0, uniq.to(tables[t].device)).cpu())
+        new_ind.append(torch.searchsorted(uniq, idx).cpu())
+    return new_tabs, torch.cat(new_ind).to(indices.dtype) if new_ind else indices.cpu()

@@ -1,0 +1,77 @@
+"""The C-ABI library builds, loads and exports every entry point of include/cb_tbe.h (CPU)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_functions():
+    with open(os.path.join(ROOT, "include", "cb_tbe.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cb_tbe_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_30656_gb300 import build, tbe
+    build.build()
+    return tbe.load_library()
+
+
+def test_header_declares_the_expected_entry_points():
+    from paper_2609_30656_gb300 import tbe
+    assert _declared_functions() == sorted(tbe.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings_and_component_names(lib):
+    from paper_2609_30656_gb300 import tbe
+    assert lib.cb_tbe_status_string(0) == b"ok"
+    assert lib.cb_tbe_status_string(7) == b"bounded device wait timed out"
+    assert tbe.component_names() == ["fwd.prep", "fwd.gather", "fwd.fixup", "bwd.keygen",
+                                     "bwd.sort", "bwd.rle", "bwd.reduce"]
+
+
+def test_host_side_argument_errors_return_before_any_gpu_work(lib):
+    from paper_2609_30656_gb300 import tbe
+    h = ctypes.c_void_p()
+    # null descriptor array / zero tables / null out pointer
+    assert lib.cb_tbe_create(None, 1, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    descs = (tbe.CbTableDesc * 1)(tbe.CbTableDesc(None, 0, 16, 0))
+    assert lib.cb_tbe_create(descs, 0, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_create(descs, 1, 0, 1, 0, None) == tbe.CB_ERR_INVALID_ARG
+    # bad pooling / index dtype / storage dtype / row size not a multiple of 16 bytes
+    assert lib.cb_tbe_create(descs, 1, 5, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_create(descs, 1, 0, 7, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    bad = (tbe.CbTableDesc * 1)(tbe.CbTableDesc(None, 0, 16, 9))
+    assert lib.cb_tbe_create(bad, 1, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    odd = (tbe.CbTableDesc * 1)(tbe.CbTableDesc(None, 0, 6, 1))  # 12-byte fp16 rows
+    assert lib.cb_tbe_create(odd, 1, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    wide = (tbe.CbTableDesc * 1)(tbe.CbTableDesc(None, 0, 1024, 1))  # dim > 512
+    assert lib.cb_tbe_create(wide, 1, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    unaligned = (tbe.CbTableDesc * 1)(tbe.CbTableDesc(8, 10, 16, 0))
+    assert lib.cb_tbe_create(unaligned, 1, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+    # calls on a null handle
+    assert lib.cb_tbe_forward(None, 1, None, 0, None, None, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_backward(None, 1, None, 0, None, None, None, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_get_error(None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_reserve(None, 1, 1) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_launch_count(None) == 0
+    lib.cb_tbe_destroy(None)
+
+
+def test_product_path_fails_loudly_without_the_library(monkeypatch, tmp_path):
+    from paper_2609_30656_gb300 import tbe
+    monkeypatch.setattr(tbe, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(tbe, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        tbe.load_library()

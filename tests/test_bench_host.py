@@ -1,0 +1,94 @@
+"""Host-side logic of bench.py: byte accounting, clock parsing, rank aggregation (CPU)."""
+
+import os
+import socket
+
+import pytest
+import torch
+import torch.multiprocessing as mp
+
+import bench
+from paper_2609_30656_gb300 import metrics, workloads as wl
+
+
+def test_forward_and_backward_bytes_by_hand():
+    # 2 tables (dims 4 and 8, fp16), batch 3, lookups 5 and 2.
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts((4, 8), 2, 3, off, weighted=True)
+    assert c.lookups_per_table == (5, 2) and c.n == 7 and c.sum_dims == 12
+    f = metrics.forward_bytes(c)
+    assert f["rows"] == 5 * 4 * 2 + 2 * 8 * 2
+    assert f["indices"] == 7 * 8 and f["offsets"] == 7 * 8 and f["weights"] == 7 * 4
+    assert f["output"] == 3 * 12 * 4
+    assert f["total"] == sum(v for k, v in f.items() if k != "total")
+    b = metrics.backward_bytes(c, [3, 1])
+    assert b["grad_gather"] == 5 * 4 * 4 + 2 * 8 * 4
+    assert b["unique_ids"] == 4 * 8 and b["grads"] == 3 * 4 * 4 + 1 * 8 * 4
+    assert metrics.forward_unique_bytes(c, [3, 1]) == f["total"] - f["rows"] + 3 * 8 + 1 * 16
+
+
+def test_radix_passes_follow_key_bits():
+    assert metrics.radix_passes([256]) == 1
+    assert metrics.radix_passes([257]) == 2
+    assert metrics.radix_passes([5_000_000] * 100) == 4   # 29-bit keys
+    assert metrics.radix_passes([100_000] * 8) == 3       # 20-bit keys
+    assert metrics.sort_bytes(10, 3) == 480
+
+
+def test_workload_description_names_the_shape():
+    d = bench.describe(wl.get_workload("cfg5"))
+    assert "100 x 5,000,000 rows" in d and "batch 65536" in d and "Zipf(1.2)" in d
+    assert "5% empty" in d and "sum pooling" in d
+    assert "weighted mean" in bench.describe(wl.get_workload("cfg4"))
+
+
+def test_clock_summary_parsing():
+    s = bench.ClockSampler(0)
+    s.out = ("1965, 2070, 900.5, Not Active, Not Active, Not Active, Active\n"
+             "1980, 2070, 950.0, Not Active, Not Active, Not Active, Not Active\n"
+             "300, 2070, 80.0, Not Active, Not Active, Not Active, Not Active\n")
+    r = s.summary()
+    assert r["sm_max_mhz"] == 2070 and r["sm_mhz"] == pytest.approx(1972.5)
+    assert r["reasons"] == ["sw_power_cap"]
+    s.out = ""
+    assert s.summary()["reasons"] == ["unsampled"]
+
+
+def test_traffic_is_null_unless_recorded_for_this_source(tmp_path, monkeypatch):
+    assert bench.recorded_traffic("fwd.gather", "no-such-workload") is None
+    assert len(bench.kernel_source_hash()) == 16
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    torch.distributed.init_process_group("gloo", rank=rank, world_size=world)
+    # rank r took (r + 1) ms and moved (r + 1) GB
+    res = bench.aggregate(float(rank + 1), 1e9 * (rank + 1), 100.0 * (rank + 1), world)
+    q.put((rank, res))
+    torch.distributed.destroy_process_group()
+
+
+def test_aggregate_takes_max_time_and_summed_work_over_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    got = dict(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for r in range(2):
+        ms, nbytes, rows = got[r]
+        assert ms == 2.0 and nbytes == 3e9 and rows == 300.0
+
+
+def test_aggregate_is_identity_on_one_rank():
+    assert bench.aggregate(1.5, 2.0, 3.0, 1) == (1.5, 2.0, 3.0)
