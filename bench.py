@@ -219,6 +219,13 @@ def sample_bytes(counts, res, rows_of_tables):
     return metrics.forward_bytes(counts)["total"] + metrics.backward_bytes(counts, uniq)["total"]
 
 
+def workload_of(args) -> wl.Workload:
+    w = wl.get_workload(args.workload)
+    if args.tables is not None and args.tables < w.num_tables:
+        w = wl.scaled(w, num_tables=args.tables, name=f"{w.name}-first{args.tables}")
+    return w
+
+
 def cpu_threads() -> int:
     try:
         return len(os.sched_getaffinity(0))
@@ -238,7 +245,7 @@ def run_ours(args):
         torch.distributed.init_process_group("nccl")
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    w = wl.get_workload(args.workload)
+    w = workload_of(args)
     seed = args.seed
     tables = wl.make_tables(w, seed, dev)
     batches = [wl.make_batch(w, seed + 1000 * rank, dev, batch_index=k) for k in range(args.rotate)]
@@ -446,7 +453,7 @@ def run_reference(args):
     if rank != 0:
         return  # rank 0 alone times the oracle
     dev = torch.device("cuda", 0) if torch.cuda.is_available() else torch.device("cpu")
-    w = wl.get_workload(args.workload)
+    w = workload_of(args)
     threads = cpu_threads()
     ntab = min(w.num_tables, args.ref_tables)
     tables = wl.make_tables(w, args.seed, dev, only=range(ntab))
@@ -499,9 +506,11 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="cfg5")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--tables", type=int, default=None,
+                    help="first N tables only (a smaller case of the same workload)")
     ap.add_argument("--rotate", type=int, default=4)
     ap.add_argument("--e2e-steps", type=int, default=5)
-    ap.add_argument("--cpu-tables", type=int, default=4)
+    ap.add_argument("--cpu-tables", type=int, default=32)
     ap.add_argument("--ref-tables", type=int, default=2)
     ap.add_argument("--ref-budget-s", type=float, default=150.0)
     ap.add_argument("--no-e2e", action="store_true")
