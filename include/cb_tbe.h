@@ -106,6 +106,30 @@ cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t 
                          const void* offsets, const float* per_sample_weights, float* out,
                          cudaStream_t stream);
 
+/* Forward without a handle and without allocating (the paper has no
+ * counterpart: this is for callers of this library that must not allocate
+ * device memory, such as a plugin running inside a framework that owns all
+ * device memory, or a steady-state loop where a cudaMalloc / cudaFree and the
+ * device-wide synchronisation it brings are not allowed).
+ * Computes exactly what cb_tbe_forward computes, with the same arguments; the
+ * table descriptors are passed per call instead of through a handle.
+ * Scratch comes from one fixed 16 MiB __device__ array inside this library,
+ * held by every GPU that loads the library until the process exits. A call
+ * needs about (n / 512 + T + 1) * (32 + 8 * max dim) bytes plus ~100 bytes per
+ * table (e.g. up to ~7.9 M lookups over 100 tables of dim 128); a larger call
+ * is refused with CB_ERR_CAPACITY before any GPU work.
+ * The first call on each device looks up the array's device address (with
+ * that device current); make that first call before any stream capture.
+ * Every call reuses the same array (its error word is cleared at the start of
+ * each call), so calls whose GPU work overlaps race: do not run two at once
+ * from several threads or streams. The call checks the offsets, synchronises
+ * `stream` and returns the device-side status (as under CB_VALIDATE). It calls
+ * no cudaMalloc, cudaFree or allocating library routine. */
+cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t num_tables, cb_pooling mode,
+                                 cb_index_dtype idx_dtype, int32_t batch, const void* indices,
+                                 int64_t num_indices, const void* offsets,
+                                 const float* per_sample_weights, float* out, cudaStream_t stream);
+
 /* Row-sparse gradient written by cb_tbe_backward. All pointers are device
  * memory owned by the caller. U = number of distinct (table, row) pairs
  * touched by the batch; F = sum over those rows of their table's dim. */

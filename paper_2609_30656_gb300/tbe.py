@@ -28,7 +28,8 @@ _IDX = {torch.int32: 0, torch.int64: 1}
 # Every entry point declared in include/cb_tbe.h.
 EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
-           "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy")
+           "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
+           "cb_tbe_forward_noalloc")
 
 
 class CbTableDesc(ctypes.Structure):
