@@ -39,6 +39,8 @@ def _deps() -> list[str]:
 
 
 def _stale() -> bool:
+    if os.environ.get("CB_TBE_NVCC_FLAGS"):
+        return True
     if not os.path.exists(LIB):
         return True
     t = os.path.getmtime(LIB)
@@ -55,6 +57,7 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
              *ARCH]
     if ptxas_info:
         flags += ["-Xptxas", "-v"]
+    flags += os.environ.get("CB_TBE_NVCC_FLAGS", "").split()
 
     def compile_one(src: str) -> tuple[str, str]:
         obj = os.path.join(BUILD_DIR, src.replace(".cu", ".o"))

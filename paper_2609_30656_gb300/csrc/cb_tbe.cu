@@ -103,6 +103,7 @@ struct cb_tbe {
     int32_t* d_bwd_class_start = nullptr;
     int* d_error = nullptr;
     uint32_t* d_never_set = nullptr;
+    uint4* d_zero_row = nullptr;  // 2 KB of zeros
     // grown on demand
     void* ws = nullptr;
     size_t ws_bytes = 0;
@@ -190,6 +191,7 @@ Problem make_problem(const cb_tbe* h, int32_t B, const void* indices, int64_t n,
                      const float* weights) {
     Problem P;
     P.tables = h->d_tables;
+    P.zero_row = h->d_zero_row;
     P.indices = indices;
     P.offsets = offsets;
     P.weights = weights;
@@ -355,6 +357,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     const size_t o_bct = off; off += align_up(sizeof(int32_t) * bct.size());
     const size_t o_bcs = off; off += align_up(sizeof(int32_t) * bcs.size());
     const size_t o_err = off; off += align_up(sizeof(int) + sizeof(uint32_t));
+    const size_t o_zero = off; off += align_up(2048);
     if (cudaMalloc(&h->persist, off) != cudaSuccess) {
         cudaGetLastError();
         delete h;
@@ -368,6 +371,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     h->d_bwd_class_start = reinterpret_cast<int32_t*>(p + o_bcs);
     h->d_error = reinterpret_cast<int*>(p + o_err);
     h->d_never_set = reinterpret_cast<uint32_t*>(p + o_err + sizeof(int));
+    h->d_zero_row = reinterpret_cast<uint4*>(p + o_zero);
     bool ok = cudaMemcpy(h->d_tables, h->tables.data(), sizeof(TableDev) * num_tables,
                          cudaMemcpyHostToDevice) == cudaSuccess;
     ok = ok && cudaMemcpy(h->d_fwd_class_tables, fct.data(), sizeof(int32_t) * fct.size(),
@@ -379,6 +383,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     ok = ok && cudaMemcpy(h->d_bwd_class_start, bcs.data(), sizeof(int32_t) * bcs.size(),
                           cudaMemcpyHostToDevice) == cudaSuccess;
     ok = ok && cudaMemset(h->d_error, 0, sizeof(int) + sizeof(uint32_t)) == cudaSuccess;
+    ok = ok && cudaMemset(h->d_zero_row, 0, 2048) == cudaSuccess;
     if (ok && (flags & CB_TIMING)) {
         for (auto& e : h->ev_fwd) ok = ok && cudaEventCreate(&e) == cudaSuccess;
         for (auto& e : h->ev_bwd) ok = ok && cudaEventCreate(&e) == cudaSuccess;

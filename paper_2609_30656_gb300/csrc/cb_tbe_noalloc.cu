@@ -132,6 +132,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
     const int64_t max_chunks = num_indices / kChunk + T + 1;
     size_t off = 0;
     const size_t o_err = off; off += up256(sizeof(int));
+    const size_t o_zero = off; off += up256(2048);
     const size_t o_tab = off; off += up256(sizeof(TableDev) * T);
     const size_t o_ct = off; off += up256(sizeof(int32_t) * T);
     const size_t o_cs = off; off += up256(sizeof(int32_t) * (nc + 1));
@@ -155,20 +156,23 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
     if (batch == 0) return CB_OK;
 
     // The array keeps the previous call's contents: upload this call's tables
-    // and class lists, and clear the error word, which must start at zero.
+    // and class lists, and clear the error word and the zero row, which must
+    // start at zero.
     std::vector<unsigned char> host(o_pos - o_tab, 0);
     memcpy(host.data(), td.data(), sizeof(TableDev) * T);
     memcpy(host.data() + (o_ct - o_tab), class_tables.data(), sizeof(int32_t) * T);
     memcpy(host.data() + (o_cs - o_tab), class_start.data(), sizeof(int32_t) * (nc + 1));
     if (cudaMemcpyAsync(base + o_tab, host.data(), host.size(), cudaMemcpyHostToDevice, stream) !=
             cudaSuccess ||
-        cudaMemsetAsync(base + o_err, 0, sizeof(int), stream) != cudaSuccess) {
+        cudaMemsetAsync(base + o_err, 0, sizeof(int), stream) != cudaSuccess ||
+        cudaMemsetAsync(base + o_zero, 0, 2048, stream) != cudaSuccess) {
         cudaGetLastError();
         return CB_ERR_CUDA;
     }
 
     Problem P;
     P.tables = reinterpret_cast<const TableDev*>(base + o_tab);
+    P.zero_row = reinterpret_cast<const uint4*>(base + o_zero);
     P.indices = indices;
     P.offsets = offsets;
     P.weights = per_sample_weights;

@@ -207,129 +207,102 @@ __global__ void __launch_bounds__(1024) bwd_finalize_kernel(Problem P, BwdOut O)
 
 template <int VPL, bool PACKED>
 struct BwdPolicy {
+    static constexpr int kDtype = CB_F32;
     static constexpr int kElems = 4;
     static constexpr int kVpl = VPL;
-    static constexpr int kUnroll = 8 / VPL;
+    static constexpr int kUnroll = CB_WALK_ROWS / VPL > 0 ? CB_WALK_ROWS / VPL : 1;
+    static constexpr bool kWeighted = PACKED;
 
-    const uint32_t* seg_start;
-    const uint32_t* vals;
-    const uint2* packed;
-    const uint32_t* uniq;
-    const float* grad_out;
-    float* grads;
-    int64_t* unique_ids;
-    int64_t* grad_offsets;
-    float* carry_head;
-    float* carry_tail;
-    int64_t* tail_owner;
-    int64_t chunk;
-    int64_t n;
-    int64_t bag_lo;
-    int64_t seg_lo;      // first unique index of this table
-    int64_t float_lo;    // first float of this table in grads
-    int32_t B;
-    int32_t sum_d;
-    int32_t doff;
+    const Problem& P;  // kernel parameters: read in place, not held in registers
+    const Plan& Q;
+    const BwdOut& O;
+    const uint4* base;  // grad_out + Doff_t, one row per bag of this table
+    int64_t float_lo;   // first float of this table in grads
+    uint32_t stride;    // sum of dims / 4
+    int32_t chunk;
+    int32_t bag_lo;
+    int32_t seg_lo;     // first unique index of this table
     int32_t dim;
-    int32_t dmax;
-    int32_t vecs;
 
-    __device__ __forceinline__ int64_t seg_begin(int64_t s) const { return __ldg(seg_start + s); }
-    __device__ __forceinline__ int64_t seg_end(int64_t s) const { return __ldg(seg_start + s + 1); }
-    __device__ __forceinline__ void item(int64_t q, int64_t& a, float& w) const {
-        const uint32_t v = __ldg(vals + q);
+    __device__ __forceinline__ int64_t seg_begin(int32_t s) const { return __ldg(O.seg_start + s); }
+    __device__ __forceinline__ int64_t seg_end(int32_t s) const { return __ldg(O.seg_start + s + 1); }
+    struct Raw {
+        uint32_t v;
+    };
+    __device__ __forceinline__ static Raw none() { return {0xffffffffu}; }
+    __device__ __forceinline__ Raw fetch(int64_t q) const { return {__ldg(O.vals_sorted + q)}; }
+    // Sorted item: the bag whose grad_out row it gathers, and w_i * s_b.
+    __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
+        int64_t bag;
         if (PACKED) {
-            if (v >= n) {  // only after an aborted sort pass: skip the item
-                a = -1;
+            if (x.v >= P.n) {  // only after an aborted sort pass: skip the item
+                a = kInvalid;
                 w = 0.f;
                 return;
             }
-            const uint2 pk = __ldg(packed + v);
-            a = pk.x;
+            const uint2 pk = __ldg(O.packed + x.v);
+            bag = pk.x;
             w = __uint_as_float(pk.y);
         } else {
-            a = v;
+            bag = x.v;
             w = 1.f;
         }
-    }
-    __device__ __forceinline__ const uint4* row(int64_t bag, bool& ok) const {
         const int64_t b = bag - bag_lo;
-        if (!ok || b < 0 || b >= B) {
-            ok = false;
-            return reinterpret_cast<const uint4*>(grad_out);
-        }
-        return reinterpret_cast<const uint4*>(grad_out + b * sum_d + doff);
+        a = (b >= 0 && b < P.B) ? static_cast<uint32_t>(b) : kInvalid;
     }
-    __device__ __forceinline__ void unpack(const uint4& x, float (&f)[4]) const {
-        cbtbe::unpack<CB_F32>(x, f);
-    }
-    __device__ __forceinline__ void emit(int64_t seg, int64_t, int64_t, bool started, bool ends,
+    __device__ __forceinline__ void emit(int32_t seg, int32_t, bool started, bool ends,
                                          float (&tot)[VPL][4], int v, bool group0) const {
         const int lane = threadIdx.x & 31;
+        const int64_t fo = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
         if (started && lane == 0) {
-            const int64_t fo = float_lo + (seg - seg_lo) * dim;
-            unique_ids[seg] = __ldg(uniq + seg);
-            grad_offsets[seg] = fo;
-            if (!ends) tail_owner[chunk] = seg;
+            O.unique_ids[seg] = __ldg(O.uniq + seg);
+            O.grad_offsets[seg] = fo;
+            if (!ends) Q.tail_owner[chunk] = seg;
         }
         if (!group0) return;
         float* dst;
-        if (started && ends) dst = grads + float_lo + (seg - seg_lo) * dim;
-        else dst = (started ? carry_tail : carry_head) + chunk * dmax;
+        if (started && ends) dst = O.grads + fo;
+        else dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
             const int vec = v + 32 * k;
-            if (vec < vecs)
+            if (vec < dim / 4)
                 reinterpret_cast<float4*>(dst)[vec] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
         }
     }
 };
 
 template <int VPL, bool PACKED>
-__global__ void __launch_bounds__(kWarpThreads) bwd_reduce_kernel(Problem P, Plan Q, BwdOut O,
-                                                                  const float* grad_out, int cls) {
+__global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
+    bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
+                      const __grid_constant__ BwdOut O, const float* grad_out, int cls) {
     if (*O.cap_fail) return;
     const int lane = threadIdx.x & 31;
     const int64_t cb = Q.class_chunk_base[cls];
-    const int64_t ce = min(Q.class_chunk_base[cls + 1], Q.max_chunks);
+    const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
     for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];
-        BwdPolicy<VPL, PACKED> pol;
-        pol.seg_start = O.seg_start;
-        pol.vals = O.vals_sorted;
-        pol.packed = O.packed;
-        pol.uniq = O.uniq;
-        pol.grad_out = grad_out;
-        pol.grads = O.grads;
-        pol.unique_ids = O.unique_ids;
-        pol.grad_offsets = O.grad_offsets;
-        pol.carry_head = Q.carry_head;
-        pol.carry_tail = Q.carry_tail;
-        pol.tail_owner = Q.tail_owner;
-        pol.chunk = j;
-        pol.n = P.n;
-        pol.bag_lo = static_cast<int64_t>(t) * P.B;
-        pol.seg_lo = O.table_first[t];
+        BwdPolicy<VPL, PACKED> pol{P, Q, O};
+        pol.base = reinterpret_cast<const uint4*>(grad_out + td.doff);
         pol.float_lo = O.float_base[t];
-        pol.B = P.B;
-        pol.sum_d = P.sum_d;
-        pol.doff = td.doff;
+        pol.stride = static_cast<uint32_t>(P.sum_d / 4);
+        pol.chunk = static_cast<int32_t>(j);
+        pol.bag_lo = t * P.B;
+        pol.seg_lo = static_cast<int32_t>(O.table_first[t]);
         pol.dim = td.dim;
-        pol.dmax = P.dmax;
-        pol.vecs = td.grad_vecs;
         ChunkCtx c;
         c.k0 = ch.k0;
-        c.k1 = ch.k0 + (ch.len & 0x7fffffffu);
-        c.first = max(ch.first, pol.seg_lo);
-        c.seg_hi = O.table_first[t + 1];
+        c.len = static_cast<int32_t>(ch.len & 0x7fffffffu);
+        c.first = static_cast<int32_t>(max64(ch.first, O.table_first[t]));
+        c.seg_hi = static_cast<int32_t>(O.table_first[t + 1]);
         c.lanes = td.grad_lanes;
         c.groups = td.grad_groups;
         c.row_vecs = td.grad_vecs;
         c.last = false;
         if (lane == 0) Q.tail_owner[j] = -1;
-        walk_chunk(pol, c, lane);
+        walk_chunk(pol, c, P.zero_row, lane);
     }
 }
 

@@ -12,60 +12,56 @@
 
 namespace cbtbe {
 
-template <int DT, int VPL>
+template <int DT, int VPL, bool WEIGHTED>
 struct FwdPolicy {
+    static constexpr int kDtype = DT;
     static constexpr int kElems = Storage<DT>::kElems;
     static constexpr int kVpl = VPL;
-    static constexpr int kUnroll = 8 / VPL;
+    static constexpr int kUnroll = CB_WALK_ROWS / VPL > 0 ? CB_WALK_ROWS / VPL : 1;
+    static constexpr bool kWeighted = WEIGHTED;
 
-    const void* offsets;
-    const void* indices;
-    const float* weights;
-    const uint4* table;
+    const Problem& P;  // kernel parameters: read in place, not held in registers
+    const Plan& Q;
     float* out;
-    float* carry_head;
-    float* carry_tail;
-    int64_t* tail_owner;
-    int* error;
+    const uint4* base;  // the table
     int64_t rows;
-    int64_t chunk;
-    int64_t bag_lo;
+    uint32_t stride;    // 16-byte vectors per row
     int32_t row_vecs;
-    int32_t is32;
-    int32_t sum_d;
+    int32_t chunk;
+    int32_t bag_lo;
     int32_t doff;
-    int32_t dmax;
-    int32_t mean;
 
-    __device__ __forceinline__ int64_t seg_begin(int64_t s) const { return load_index(offsets, s, is32); }
-    __device__ __forceinline__ int64_t seg_end(int64_t s) const { return load_index(offsets, s + 1, is32); }
-    __device__ __forceinline__ void item(int64_t q, int64_t& a, float& w) const {
-        a = load_index(indices, q, is32);
-        w = weights ? __ldg(weights + q) : 1.f;
+    __device__ __forceinline__ int64_t seg_begin(int32_t s) const { return load_index(P.offsets, s, P.is32); }
+    __device__ __forceinline__ int64_t seg_end(int32_t s) const { return load_index(P.offsets, s + 1, P.is32); }
+    struct Raw {
+        int64_t r;
+        float w;
+    };
+    __device__ __forceinline__ static Raw none() { return {-1, 0.f}; }
+    __device__ __forceinline__ Raw fetch(int64_t q) const {
+        return {load_index(P.indices, q, P.is32), WEIGHTED ? __ldg(P.weights + q) : 1.f};
     }
-    __device__ __forceinline__ const uint4* row(int64_t r, bool& ok) const {
-        if (!ok) return table;
-        if (r < 0 || r >= rows) {
-            set_error(error, CB_ERR_INDEX_OOB);  // contributes nothing
-            ok = false;
-            return table;
+    // Row id of a lookup, checked once here; an out-of-range id contributes nothing.
+    __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
+        w = x.w;
+        if (x.r < 0 || x.r >= rows) {
+            set_error(P.error, CB_ERR_INDEX_OOB);
+            a = kInvalid;
+        } else {
+            a = static_cast<uint32_t>(x.r);
         }
-        return table + r * row_vecs;
     }
-    __device__ __forceinline__ void unpack(const uint4& x, float (&f)[kElems]) const {
-        cbtbe::unpack<DT>(x, f);
-    }
-    __device__ __forceinline__ void emit(int64_t bag, int64_t s, int64_t e, bool started, bool ends,
+    __device__ __forceinline__ void emit(int32_t bag, int32_t L, bool started, bool ends,
                                          float (&tot)[VPL][kElems], int v, bool group0) const {
-        if (started && !ends && (threadIdx.x & 31) == 0) tail_owner[chunk] = bag;
+        if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = bag;
         if (!group0) return;
         float* dst;
-        float L = 0.f;
+        float scale = 0.f;
         if (started && ends) {
-            dst = out + (bag - bag_lo) * sum_d + doff;
-            if (mean && e > s) L = static_cast<float>(e - s);
+            dst = out + static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff;
+            if (P.mean && L > 0) scale = static_cast<float>(L);
         } else {
-            dst = (started ? carry_tail : carry_head) + chunk * dmax;
+            dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
         }
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
@@ -73,7 +69,7 @@ struct FwdPolicy {
             if (vec >= row_vecs) continue;
             float o[kElems];
 #pragma unroll
-            for (int x = 0; x < kElems; ++x) o[x] = L > 0.f ? tot[k][x] / L : tot[k][x];
+            for (int x = 0; x < kElems; ++x) o[x] = scale > 0.f ? tot[k][x] / scale : tot[k][x];
             float4* d4 = reinterpret_cast<float4*>(dst + vec * kElems);
 #pragma unroll
             for (int x = 0; x < kElems / 4; ++x)
@@ -82,45 +78,35 @@ struct FwdPolicy {
     }
 };
 
-template <int DT, int VPL>
-__global__ void __launch_bounds__(kWarpThreads) fwd_gather_kernel(Problem P, Plan Q, float* out,
-                                                                  int cls) {
+template <int DT, int VPL, bool WEIGHTED>
+__global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
+    fwd_gather_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q, float* out,
+                      int cls) {
     const int lane = threadIdx.x & 31;
     const int64_t cb = Q.class_chunk_base[cls];
-    const int64_t ce = min(Q.class_chunk_base[cls + 1], Q.max_chunks);
+    const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
     for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
         const Chunk ch = Q.chunks[j];
         const TableDev& td = P.tables[ch.table];
-        FwdPolicy<DT, VPL> pol;
-        pol.offsets = P.offsets;
-        pol.indices = P.indices;
-        pol.weights = P.weights;
-        pol.table = static_cast<const uint4*>(td.data);
-        pol.out = out;
-        pol.carry_head = Q.carry_head;
-        pol.carry_tail = Q.carry_tail;
-        pol.tail_owner = Q.tail_owner;
-        pol.error = P.error;
+        FwdPolicy<DT, VPL, WEIGHTED> pol{P, Q, out};
+        pol.base = static_cast<const uint4*>(td.data);
         pol.rows = td.rows;
-        pol.chunk = j;
-        pol.bag_lo = static_cast<int64_t>(ch.table) * P.B;
+        pol.stride = static_cast<uint32_t>(td.row_vecs);
         pol.row_vecs = td.row_vecs;
-        pol.is32 = P.is32;
-        pol.sum_d = P.sum_d;
+        pol.chunk = static_cast<int32_t>(j);
+        pol.bag_lo = ch.table * P.B;
         pol.doff = td.doff;
-        pol.dmax = P.dmax;
-        pol.mean = P.mean;
         ChunkCtx c;
         c.k0 = ch.k0;
-        c.k1 = ch.k0 + (ch.len & 0x7fffffffu);
-        c.first = ch.first;
+        c.len = static_cast<int32_t>(ch.len & 0x7fffffffu);
+        c.first = static_cast<int32_t>(ch.first);
         c.seg_hi = pol.bag_lo + P.B;
         c.lanes = td.lanes;
         c.groups = td.groups;
         c.row_vecs = td.row_vecs;
         c.last = (ch.len >> 31) != 0;
         if (lane == 0) Q.tail_owner[j] = -1;
-        walk_chunk(pol, c, lane);
+        walk_chunk(pol, c, P.zero_row, lane);
     }
 }
 
@@ -161,11 +147,11 @@ __global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(Problem P, Plan
     }
 }
 
-template <int DT, int VPL>
+template <int DT, int VPL, bool W>
 static int gather_grid(int num_sms) {
     static int per_sm = -1;
     if (per_sm < 0) {
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fwd_gather_kernel<DT, VPL>,
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fwd_gather_kernel<DT, VPL, W>,
                                                           kWarpThreads, 0) != cudaSuccess ||
             per_sm < 1)
             per_sm = 1;
@@ -177,8 +163,13 @@ template <int DT, int VPL>
 static void launch_one(const Problem& P, const Plan& Q, float* out, int cls, int64_t chunk_bound,
                        int num_sms, cudaStream_t s) {
     const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
-    const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL>(num_sms)));
-    fwd_gather_kernel<DT, VPL><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
+    if (P.weights) {
+        const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL, true>(num_sms)));
+        fwd_gather_kernel<DT, VPL, true><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
+    } else {
+        const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL, false>(num_sms)));
+        fwd_gather_kernel<DT, VPL, false><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
+    }
 }
 
 void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,

@@ -25,6 +25,12 @@ namespace cbtbe {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kWarpThreads = 256;  // block size of the warp-per-chunk kernels
+#ifndef CB_WALK_MIN_BLOCKS
+#define CB_WALK_MIN_BLOCKS 4  // resident blocks per SM the walker kernels are compiled for
+#endif
+#ifndef CB_WALK_ROWS
+#define CB_WALK_ROWS 4  // 16-byte rows in flight per lane in the walker (with one vector per lane)
+#endif
 constexpr int64_t kNoSeg = INT64_MAX;
 
 // Per-table facts the kernels need, built once at create time.
@@ -56,6 +62,7 @@ struct Chunk {
 
 struct Problem {
     const TableDev* tables;
+    const uint4* zero_row;  // 2 KB of zeros: the row an invalid or padding item reads
     const void* indices;
     const void* offsets;
     const float* weights;
@@ -143,156 +150,236 @@ __device__ __forceinline__ void unpack<CB_BF16>(const uint4& r, float (&f)[8]) {
     }
 }
 
+// ---------------------------------------------------------------- accumulation
+
+// acc += w * row (WEIGHTED) or acc += row. Half-precision rows use the
+// mixed-precision add of sm_100+ (f16/bf16 operand widened exactly, fp32 sum),
+// which is the same arithmetic as widening first and then adding.
+template <int DT, bool WEIGHTED>
+__device__ __forceinline__ void accumulate(float (&a)[Storage<DT>::kElems], const uint4& x, float w) {
+    const uint32_t word[4] = {x.x, x.y, x.z, x.w};
+    if constexpr (DT == CB_F32) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float f = __uint_as_float(word[i]);
+            a[i] = WEIGHTED ? fmaf(w, f, a[i]) : a[i] + f;
+        }
+    } else if constexpr (WEIGHTED) {
+        float f[8];
+        unpack<DT>(x, f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a[i] = fmaf(w, f[i], a[i]);
+    } else if constexpr (DT == CB_F16) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            asm("{ .reg .b16 lo, hi;\n\t mov.b32 {lo, hi}, %2;\n\t"
+                " add.rn.f32.f16 %0, lo, %0;\n\t add.rn.f32.f16 %1, hi, %1; }"
+                : "+f"(a[2 * i]), "+f"(a[2 * i + 1]) : "r"(word[i]));
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            asm("{ .reg .b16 lo, hi;\n\t mov.b32 {lo, hi}, %2;\n\t"
+                " add.rn.f32.bf16 %0, lo, %0;\n\t add.rn.f32.bf16 %1, hi, %1; }"
+                : "+f"(a[2 * i]), "+f"(a[2 * i + 1]) : "r"(word[i]));
+    }
+}
+
 // ---------------------------------------------------------------- the walker
 //
 // Pol (policy) supplies:
-//   kElems, kVpl (16-byte vectors per lane), kUnroll (items in flight per lane)
-//   int64_t seg_end(int64_t s)          end position of segment s (s < seg_hi)
-//   void item(int64_t q, int64_t& a, float& w)   payload of item q (lane-local)
-//   const uint4* row(int64_t a, bool& ok)         row of an item (ok=false: skip)
-//   void unpack(const uint4&, float (&)[kElems])
-//   void emit(seg, s, e, started, ends, tot, lane-in-group v, is_group0)
+//   kDtype, kElems, kVpl (16-byte vectors per lane), kUnroll (rows in flight per
+//   lane), kWeighted
+//   int64_t seg_begin(s), seg_end(s)    positions of segment s (s < seg_hi)
+//   Raw fetch(q), static Raw none()      raw payload of item q (loads only)
+//   void decode(Raw, uint32_t& a, float& w)  row number within `base`
+//                                            (kInvalid = skip) and coefficient
+//   const uint4* base; uint32_t stride       row a starts at base + a * stride
+//   void emit(seg, len, started, ends, tot, lane-in-group v, is_group0)
+//                                            len = segment length when complete
+// Positions inside the walker are relative to the chunk start and clamped to
+// [kRelLo, kRelHi], which keeps every comparison with [0, len] exact in 32 bits.
 // The segment range of the chunk is [first, seg_hi); segments that start at or
 // after the chunk end belong to the next chunk, except after the last chunk of a
 // table (trailing empty bags), which `last` allows.
 
+constexpr uint32_t kInvalid = 0xffffffffu;
+constexpr int32_t kRelLo = -1;
+constexpr int32_t kRelHi = 1 << 30;
+
 struct ChunkCtx {
-    int64_t k0, k1;       // item positions [k0, k1)
-    int64_t first;        // first segment
-    int64_t seg_hi;       // segments of this table end before seg_hi
-    int32_t lanes;        // V
-    int32_t groups;       // G
-    int32_t row_vecs;     // vectors per row
-    bool last;            // owns trailing segments that start at k1
+    int64_t k0;        // absolute position of the chunk's first item
+    int32_t len;       // items in the chunk
+    int32_t first;     // first segment
+    int32_t seg_hi;    // segments of this table end before seg_hi
+    int32_t lanes;     // V
+    int32_t groups;    // G
+    int32_t row_vecs;  // vectors per row
+    bool last;         // owns trailing segments that start at the chunk end
 };
 
+__device__ __forceinline__ int32_t rel_pos(int64_t x, int64_t k0) {
+    const int64_t r = x - k0;
+    return r < kRelLo ? kRelLo : (r > kRelHi ? kRelHi : static_cast<int32_t>(r));
+}
+
 template <class Pol>
-__device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, int lane) {
+__device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const uint4* zero_row,
+                                           int lane) {
     constexpr int E = Pol::kElems;
     constexpr int VPL = Pol::kVpl;
     constexpr int U = Pol::kUnroll;
+    constexpr bool W = Pol::kWeighted;
     const int V = c.lanes, G = c.groups;
     const int g = lane / V;
     const int v = lane - g * V;
-    const bool active = g < G;
+    const int ustop = min(U, 32 / G);  // row groups per step
+    const int step = ustop * G;        // items per step (<= 32, divides 32)
+    const int32_t len = c.len;
+    // Lanes past the row (non power-of-two rows) and vectors past it read zeros.
+    const uint4* vzero[VPL];
+    bool vlive[VPL];
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) {
+        vlive[k] = g < G && v + 32 * k < c.row_vecs;
+        vzero[k] = zero_row + (v + 32 * k) % 128;
+    }
 
-    // Segment-end window: lane i holds the end of segment win_base + i.
-    int64_t win_base = c.first;
-    int64_t my_end = (win_base + lane < c.seg_hi) ? pol.seg_end(win_base + lane) : kNoSeg;
-    int64_t seg = c.first;
-    int64_t s_cur = kNoSeg, e_cur = kNoSeg;
+    // Segment-end window: lane i holds the (relative) end of segment win + i.
+    int32_t win = c.first;
+    int32_t my_end = (win + lane < c.seg_hi) ? rel_pos(pol.seg_end(win + lane), c.k0) : kRelHi;
+    int32_t seg = c.first;
+    int32_t s_cur = kRelHi, e_cur = kRelHi;
     if (seg < c.seg_hi) {
-        s_cur = pol.seg_begin(seg);
+        s_cur = rel_pos(pol.seg_begin(seg), c.k0);
         e_cur = __shfl_sync(kFull, my_end, 0);
     }
 
-    float ain[VPL][E], aout[VPL][E];
+    // fp32 rows (tables or gradients) sum in two levels (see the fold below);
+    // half-precision rows, whose tolerance is far looser, use one level, which
+    // frees registers for occupancy.
+    constexpr bool kTwoLevel = Pol::kDtype == CB_F32;
+    float ain[VPL][E], aout[VPL][kTwoLevel ? E : 1];
 #pragma unroll
-    for (int k = 0; k < VPL; ++k)
+    for (int k = 0; k < VPL; ++k) {
 #pragma unroll
-        for (int x = 0; x < E; ++x) ain[k][x] = aout[k][x] = 0.f;
+        for (int x = 0; x < E; ++x) ain[k][x] = 0.f;
+#pragma unroll
+        for (int x = 0; x < (kTwoLevel ? E : 1); ++x) aout[k][x] = 0.f;
+    }
 
     auto flush = [&]() {
         float tot[VPL][E];
 #pragma unroll
         for (int k = 0; k < VPL; ++k)
 #pragma unroll
-            for (int x = 0; x < E; ++x) tot[k][x] = aout[k][x] + ain[k][x];
+            for (int x = 0; x < E; ++x) tot[k][x] = kTwoLevel ? aout[k][x] + ain[k][x] : ain[k][x];
         for (int off = V; off < V * G; off <<= 1) {
 #pragma unroll
             for (int k = 0; k < VPL; ++k)
 #pragma unroll
                 for (int x = 0; x < E; ++x) tot[k][x] += __shfl_xor_sync(kFull, tot[k][x], off);
         }
-        pol.emit(seg, s_cur, e_cur, s_cur >= c.k0, e_cur <= c.k1, tot, v, g == 0);
+        pol.emit(seg, e_cur - s_cur, s_cur >= 0, e_cur <= len, tot, v, g == 0);
 #pragma unroll
-        for (int k = 0; k < VPL; ++k)
+        for (int k = 0; k < VPL; ++k) {
 #pragma unroll
-            for (int x = 0; x < E; ++x) ain[k][x] = aout[k][x] = 0.f;
+            for (int x = 0; x < E; ++x) ain[k][x] = 0.f;
+#pragma unroll
+            for (int x = 0; x < (kTwoLevel ? E : 1); ++x) aout[k][x] = 0.f;
+        }
     };
     auto advance = [&]() {
         ++seg;
         s_cur = e_cur;
         if (seg >= c.seg_hi) {
-            s_cur = e_cur = kNoSeg;
+            s_cur = e_cur = kRelHi;
             return;
         }
-        if (seg - win_base >= 32) {
-            win_base = seg;
-            my_end = (win_base + lane < c.seg_hi) ? pol.seg_end(win_base + lane) : kNoSeg;
+        if (seg - win >= 32) {
+            win = seg;
+            my_end = (win + lane < c.seg_hi) ? rel_pos(pol.seg_end(win + lane), c.k0) : kRelHi;
         }
-        e_cur = __shfl_sync(kFull, my_end, static_cast<int>(seg - win_base));
+        e_cur = __shfl_sync(kFull, my_end, seg - win);
     };
 
-    int64_t nxt_a = 0;
-    float nxt_w = 1.f;
-    if (c.k0 + lane < c.k1) pol.item(c.k0 + lane, nxt_a, nxt_w);
+    typename Pol::Raw nxt = Pol::none();
+    if (lane < len) nxt = pol.fetch(c.k0 + lane);
 
-    for (int64_t base = c.k0; base < c.k1; base += 32) {
-        const int nb = static_cast<int>(min64(32, c.k1 - base));
-        const int64_t my_a = nxt_a;
-        const float my_w = nxt_w;
-        // Prefetch the next batch's payload while this batch's rows are in flight.
-        nxt_a = 0;
-        nxt_w = 1.f;
-        if (base + 32 + lane < c.k1) pol.item(base + 32 + lane, nxt_a, nxt_w);
+    for (int32_t base = 0; base < len; base += 32) {
+        const int nb = min(32, len - base);
+        const typename Pol::Raw cur = nxt;
+        // Prefetch the next batch's raw payload while this batch's rows are in
+        // flight; it is only decoded when its batch comes up.
+        nxt = Pol::none();
+        if (base + 32 + lane < len) nxt = pol.fetch(c.k0 + base + 32 + lane);
+        uint32_t my_a = kInvalid;  // lanes >= nb hold kInvalid
+        float my_w = 0.f;
+        if (lane < nb) pol.decode(cur, my_a, my_w);
 
-        for (int i0 = 0; i0 < nb; i0 += U * G) {
+        for (int i0 = 0; i0 < nb; i0 += step) {
+            // Issue every row load of the step first; an invalid or padding item
+            // reads the zero row, so it adds nothing and needs no bookkeeping.
             uint4 buf[U][VPL];
+            float wt[U];
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int i = i0 + u * G + g;
-                const int64_t a = __shfl_sync(kFull, my_a, i & 31);
-                bool ok = active && i < nb;
-                const uint4* rp = pol.row(a, ok);
+                const uint32_t a = __shfl_sync(kFull, my_a, i & 31);
+                wt[u] = W ? __shfl_sync(kFull, my_w, i & 31) : 1.f;
+                const bool ok = u < ustop && a != kInvalid;
+                const uint4* rp = pol.base + static_cast<size_t>(a) * pol.stride;
 #pragma unroll
-                for (int k = 0; k < VPL; ++k) {
-                    const int vec = v + k * 32;
-                    buf[u][k] = (ok && vec < c.row_vecs) ? __ldg(rp + vec) : make_uint4(0, 0, 0, 0);
-                }
+                for (int k = 0; k < VPL; ++k)
+                    buf[u][k] = __ldg((ok && vlive[k]) ? rp + v + 32 * k : vzero[k]);
             }
+            // Then add them in position order, emitting segments as they end.
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int ifirst = i0 + u * G;
                 if (ifirst >= nb) break;
-                const int i = ifirst + g;
-                const float w = __shfl_sync(kFull, my_w, i & 31);
-                const int64_t q = base + i;
-                const int64_t qmax = base + min(ifirst + G, nb) - 1;
-                bool added = !(active && i < nb);
-                while (true) {
-                    if (!added && q < e_cur) {
+                const int32_t qlast = base + min(ifirst + G, nb) - 1;  // last item of this row group
+                if (e_cur > qlast) {
 #pragma unroll
-                        for (int k = 0; k < VPL; ++k) {
-                            float f[E];
-                            pol.unpack(buf[u][k], f);
+                    for (int k = 0; k < VPL; ++k) accumulate<Pol::kDtype, W>(ain[k], buf[u][k], wt[u]);
+                } else {
+                    // One or more segments end inside this row group.
+                    const int32_t q = base + ifirst + g;
+                    bool added = false;
+                    do {
+                        if (!added && q < e_cur) {
 #pragma unroll
-                            for (int x = 0; x < E; ++x) ain[k][x] = fmaf(w, f[x], ain[k][x]);
+                            for (int k = 0; k < VPL; ++k)
+                                accumulate<Pol::kDtype, W>(ain[k], buf[u][k], wt[u]);
+                            added = true;
                         }
-                        added = true;
+                        flush();
+                        advance();
+                    } while (e_cur <= qlast);
+                    if (!added) {
+#pragma unroll
+                        for (int k = 0; k < VPL; ++k) accumulate<Pol::kDtype, W>(ain[k], buf[u][k], wt[u]);
                     }
-                    if (e_cur > qmax) break;
-                    flush();
-                    advance();
                 }
             }
         }
         // Two-level summation: at most 32 / G terms per lane enter `ain` before
         // it is folded into `aout`, which bounds the fp32 rounding error.
+        if (kTwoLevel) {
 #pragma unroll
-        for (int k = 0; k < VPL; ++k)
+            for (int k = 0; k < VPL; ++k)
 #pragma unroll
-            for (int x = 0; x < E; ++x) {
-                aout[k][x] += ain[k][x];
-                ain[k][x] = 0.f;
-            }
+                for (int x = 0; x < E; ++x) {
+                    aout[k][x] += ain[k][x];
+                    ain[k][x] = 0.f;
+                }
+        }
     }
 
     // Segments still open at the chunk end: finish those that end here, emit the
     // piece of the one that continues, and (last chunk only) the trailing empties.
     while (seg < c.seg_hi) {
-        if (!c.last && s_cur >= c.k1) break;
-        const bool done = e_cur <= c.k1;
+        if (!c.last && s_cur >= len) break;
+        const bool done = e_cur <= len;
         flush();
         if (!done) break;
         advance();
