@@ -43,9 +43,13 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
             const bool valid = q < k1;
             int64_t my_bag = -1, my_s = 0, my_e = 0;
             while (true) {
+                // Ends in the window never decrease (valid offsets), so the number
+                // of bags of the window that end at or before q is a binary search.
                 int cnt = 0;
 #pragma unroll
-                for (int i = 0; i < 32; ++i) cnt += (__shfl_sync(kFull, my_end, i) <= q) ? 1 : 0;
+                for (int b = 16; b >= 1; b >>= 1)
+                    if (__shfl_sync(kFull, my_end, cnt + b - 1) <= q) cnt += b;
+                if (__shfl_sync(kFull, my_end, 31) <= q) cnt = 32;
                 const int64_t e_sel = __shfl_sync(kFull, my_end, cnt < 32 ? cnt : 31);
                 const int64_t s_sel = __shfl_sync(kFull, my_end, cnt > 0 ? cnt - 1 : 0);
                 if (valid && my_bag < 0 && cnt < 32) {

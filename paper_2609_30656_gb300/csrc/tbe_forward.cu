@@ -63,17 +63,20 @@ struct FwdPolicy {
         } else {
             dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
         }
+        if (scale > 0.f) {  // mean pooling of a complete, non-empty bag
+#pragma unroll
+            for (int k = 0; k < VPL; ++k)
+#pragma unroll
+                for (int x = 0; x < kElems; ++x) tot[k][x] = tot[k][x] / scale;
+        }
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
             const int vec = v + 32 * k;
             if (vec >= row_vecs) continue;
-            float o[kElems];
-#pragma unroll
-            for (int x = 0; x < kElems; ++x) o[x] = scale > 0.f ? tot[k][x] / scale : tot[k][x];
             float4* d4 = reinterpret_cast<float4*>(dst + vec * kElems);
 #pragma unroll
             for (int x = 0; x < kElems / 4; ++x)
-                d4[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+                d4[x] = make_float4(tot[k][4 * x], tot[k][4 * x + 1], tot[k][4 * x + 2], tot[k][4 * x + 3]);
         }
     }
 };

@@ -333,6 +333,14 @@ __device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const ui
                     buf[u][k] = __ldg((ok && vlive[k]) ? rp + v + 32 * k : vzero[k]);
             }
             // Then add them in position order, emitting segments as they end.
+            if (i0 + step <= nb && e_cur > base + i0 + step - 1) {
+                // Common case: a full step inside the current segment.
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+#pragma unroll
+                    for (int k = 0; k < VPL; ++k) accumulate<Pol::kDtype, W>(ain[k], buf[u][k], wt[u]);
+                continue;
+            }
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int ifirst = i0 + u * G;
