@@ -214,7 +214,7 @@ struct BwdPolicy {
     static constexpr int kDtype = CB_F32;
     static constexpr int kElems = 4;
     static constexpr int kVpl = VPL;
-    static constexpr int kUnroll = CB_WALK_ROWS / VPL > 0 ? CB_WALK_ROWS / VPL : 1;
+    static constexpr int kUnroll = CB_REDUCE_ROWS / VPL > 0 ? CB_REDUCE_ROWS / VPL : 1;
     static constexpr bool kWeighted = PACKED;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
@@ -277,7 +277,7 @@ struct BwdPolicy {
 };
 
 template <int VPL, bool PACKED>
-__global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
+__global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
     bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
                       const __grid_constant__ BwdOut O, const float* grad_out, int cls) {
     if (*O.cap_fail) return;

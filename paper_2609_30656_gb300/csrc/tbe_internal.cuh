@@ -31,6 +31,12 @@ constexpr int kWarpThreads = 256;  // block size of the warp-per-chunk kernels
 #ifndef CB_WALK_ROWS
 #define CB_WALK_ROWS 4  // 16-byte rows in flight per lane in the walker (with one vector per lane)
 #endif
+#ifndef CB_REDUCE_MIN_BLOCKS
+#define CB_REDUCE_MIN_BLOCKS 3  // the backward reduce's own targets (from the same sweep)
+#endif
+#ifndef CB_REDUCE_ROWS
+#define CB_REDUCE_ROWS 8
+#endif
 constexpr int64_t kNoSeg = INT64_MAX;
 
 // Per-table facts the kernels need, built once at create time.

@@ -36,10 +36,14 @@ __device__ __forceinline__ void store_volatile(uint32_t* p, uint32_t v) {
     *reinterpret_cast<volatile uint32_t*>(p) = v;
 }
 
-__global__ void __launch_bounds__(kSortThreads) onesweep_kernel(SortPass S) {
-    __shared__ uint32_t sh_keys[kSortTile];
-    __shared__ uint32_t sh_vals[kSortTile];
-    __shared__ uint32_t sh_warp[kSortWarps][kRadix];  // per-warp counts, then prefixes
+constexpr int kLookbackWindow = 8;  // predecessor tiles inspected per look-back round
+
+__global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
+    extern __shared__ __align__(16) uint32_t sh_dyn[];
+    uint32_t* sh_keys = sh_dyn;                        // tile-sorted keys
+    uint32_t* sh_vals = sh_dyn + kSortTile;            // tile-sorted payloads
+    uint32_t* sh_vals_in = sh_dyn + 2 * kSortTile;     // payloads in load order
+    __shared__ uint32_t sh_warp[kSortWarps][kRadix];   // per-warp counts, then prefixes
     __shared__ uint32_t sh_start[kRadix];              // tile-local start of each digit
     __shared__ long long sh_goff[kRadix];              // global destination - local index
     __shared__ int64_t sh_scan[33];
@@ -58,28 +62,30 @@ __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(SortPass S) {
     const int tile_count = static_cast<int>(min64(kSortTile, S.n - tile_base));
 
     // Warp-striped load: item j of lane l is position tile_base + wid*512 + j*32 + l.
-    uint32_t key[kSortItems], val[kSortItems];
-    uint32_t rank[kSortItems];
-    const uint32_t lt_mask = (1u << lane) - 1u;
+    // Payloads wait in shared memory; keys and ranks stay in registers.
+    uint32_t key[kSortItems];
+    uint32_t rank2[kSortItems / 2];  // two 16-bit ranks per register
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         const bool valid = local < tile_count;
         key[j] = valid ? __ldg(S.keys_in + tile_base + local) : 0xffffffffu;
-        val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
+        if (valid) sh_vals_in[local] = __ldg(S.vals_in + tile_base + local);
     }
+    const uint32_t lt_mask = (1u << lane) - 1u;
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         const bool valid = local < tile_count;
         const uint32_t vmask = __ballot_sync(kFull, valid);
         const uint32_t d = (key[j] >> S.shift) & (kRadix - 1);
-        uint32_t peers = 0, before = 0;
+        uint32_t peers = 0, before = 0, r = 0;
         if (valid) {
             peers = __match_any_sync(vmask, d);
             before = sh_warp[wid][d];
-            rank[j] = before + __popc(peers & lt_mask);
+            r = before + __popc(peers & lt_mask);
         }
+        if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;
         __syncwarp();
         if (valid && lane == __ffs(peers) - 1) sh_warp[wid][d] = before + __popc(peers);
         __syncwarp();
@@ -96,39 +102,47 @@ __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(SortPass S) {
         count += c;
     }
     uint32_t* my_status = S.status + static_cast<int64_t>(tile) * kRadix + d;
-    if (tile == 0) {
-        store_volatile(my_status, kFlagIncl | count);
-    } else {
-        store_volatile(my_status, kFlagAgg | count);
-    }
+    store_volatile(my_status, (tile == 0 ? kFlagIncl : kFlagAgg) | count);
     int64_t total;
     const int64_t start = block_excl_scan(count, sh_scan, &total);
     sh_start[d] = static_cast<uint32_t>(start);
 
-    // Decoupled look-back over earlier tiles for digit d.
+    // Decoupled look-back over earlier tiles for digit d, kLookbackWindow
+    // predecessors per round (independent loads), bounded in time.
     uint32_t excl = 0;
     if (tile > 0) {
         int64_t k = static_cast<int64_t>(tile) - 1;
         const uint64_t t0 = global_ns();
         uint32_t spins = 0;
-        while (true) {
-            const uint32_t* src = (S.force_timeout && tile == 1)
-                                      ? S.never_set
-                                      : S.status + k * kRadix + d;
-            const uint32_t word = load_volatile(src);
-            const uint32_t flag = word & ~kCountMask;
-            if (flag == 0) {
+        bool done = false;
+        while (!done) {
+            uint32_t word[kLookbackWindow];
+#pragma unroll
+            for (int w = 0; w < kLookbackWindow; ++w) {
+                const int64_t kk = k - w;
+                const uint32_t* src = (S.force_timeout && tile == 1) ? S.never_set
+                                                                      : S.status + kk * kRadix + d;
+                word[w] = kk >= 0 ? load_volatile(src) : kFlagIncl;
+            }
+            int used = 0;
+#pragma unroll
+            for (int w = 0; w < kLookbackWindow; ++w) {
+                if (done || used < w) continue;      // stopped earlier in this round
+                const uint32_t flag = word[w] & ~kCountMask;
+                if (flag == 0) continue;             // not published yet: poll it again
+                excl += word[w] & kCountMask;
+                used = w + 1;
+                if (flag == kFlagIncl || k - w == 0) done = true;
+            }
+            k -= used;
+            if (!done && used == 0) {
                 if ((++spins & 63u) == 0 && global_ns() - t0 > S.timeout_ns) {
                     set_error(S.error, CB_ERR_TIMEOUT);
                     atomicExch(&sh_abort, 1);
                     break;
                 }
                 __nanosleep(32);
-                continue;
             }
-            excl += word & kCountMask;
-            if (flag == kFlagIncl || k == 0) break;
-            --k;
         }
         store_volatile(my_status, kFlagIncl | ((excl + count) & kCountMask));
     }
@@ -141,9 +155,10 @@ __global__ void __launch_bounds__(kSortThreads) onesweep_kernel(SortPass S) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         if (local < tile_count) {
             const uint32_t dd = (key[j] >> S.shift) & (kRadix - 1);
-            const uint32_t pos = sh_start[dd] + sh_warp[wid][dd] + rank[j];
+            const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
+            const uint32_t pos = sh_start[dd] + sh_warp[wid][dd] + r;
             sh_keys[pos] = key[j];
-            sh_vals[pos] = val[j];
+            sh_vals[pos] = sh_vals_in[local];
         }
     }
     __syncthreads();
@@ -174,9 +189,16 @@ void launch_digit_scan(const uint32_t* hist, uint32_t* base, int passes, cudaStr
     digit_scan_kernel<<<passes, kRadix, 0, s>>>(hist, base);
 }
 
+constexpr int kSortDynSmem = 3 * kSortTile * sizeof(uint32_t);  // 48 KB
+
 void launch_onesweep(const SortPass& S, cudaStream_t s) {
+    static bool configured = false;
+    if (!configured) {
+        cudaFuncSetAttribute(onesweep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSortDynSmem);
+        configured = true;
+    }
     const int64_t tiles = sort_num_tiles(S.n);
-    onesweep_kernel<<<static_cast<unsigned>(tiles), kSortThreads, 0, s>>>(S);
+    onesweep_kernel<<<static_cast<unsigned>(tiles), kSortThreads, kSortDynSmem, s>>>(S);
 }
 
 }  // namespace cbtbe
