@@ -84,13 +84,18 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
                 }
             }
             // Digit histograms of every pass (warp-aggregated shared atomics).
+            // Digits that all lanes share (the high digits, inside one table)
+            // cost one shared atomic; the others one atomic per lane.
             const uint32_t vmask = __ballot_sync(kFull, valid);
-            if (valid) {
-                const uint32_t key = K.keys[q];
-                for (int p = 0; p < K.passes; ++p) {
-                    const uint32_t dgt = (key >> (8 * p)) & 255u;
-                    const uint32_t peers = __match_any_sync(vmask, dgt);
-                    if (lane == __ffs(peers) - 1) atomicAdd(&sh_hist[p * 256 + dgt], __popc(peers));
+            const uint32_t key = valid ? K.keys[q] : 0u;
+            const int leader = __ffs(vmask) - 1;
+            for (int p = 0; p < K.passes; ++p) {
+                const uint32_t dgt = (key >> (8 * p)) & 255u;
+                const uint32_t d0 = __shfl_sync(kFull, dgt, leader);
+                if (__all_sync(kFull, !valid || dgt == d0)) {
+                    if (lane == leader) atomicAdd(&sh_hist[p * 256 + d0], __popc(vmask));
+                } else if (valid) {
+                    atomicAdd(&sh_hist[p * 256 + dgt], 1u);
                 }
             }
         }
@@ -312,35 +317,26 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
 
 // ---------------------------------------------------------------- (6) fix-up
 
-__global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(Problem P, Plan Q, BwdOut O) {
+__global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(const __grid_constant__ Problem P,
+                                                                 const __grid_constant__ Plan Q,
+                                                                 const __grid_constant__ BwdOut O) {
     if (*O.cap_fail) return;
     const int lane = threadIdx.x & 31;
-    const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
-    for (int64_t j = warp_id_global(); j < total; j += warps_in_grid()) {
-        const int64_t seg = Q.tail_owner[j];
-        if (seg < 0) continue;
-        const int t = Q.chunks[j].table;
-        const TableDev& td = P.tables[t];
-        const int64_t e = O.seg_start[seg + 1];
-        float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
-        for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
-            const float4 a = *reinterpret_cast<const float4*>(Q.carry_tail + j * P.dmax + x0);
-            double acc[4] = {a.x, a.y, a.z, a.w};
-            for (int64_t jj = j + 1; jj < total; ++jj) {
-                const Chunk c2 = Q.chunks[jj];
-                if (c2.table != t || c2.first != seg || c2.k0 >= e) break;
-                const float4 h = *reinterpret_cast<const float4*>(Q.carry_head + jj * P.dmax + x0);
-                acc[0] += h.x;
-                acc[1] += h.y;
-                acc[2] += h.z;
-                acc[3] += h.w;
-                if (e <= c2.k0 + static_cast<int64_t>(c2.len & 0x7fffffffu)) break;
-            }
-            *reinterpret_cast<float4*>(dst + x0) =
-                make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
-                            static_cast<float>(acc[2]), static_cast<float>(acc[3]));
-        }
-    }
+    const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    const int64_t j = warp_id_global();
+    if (j >= total) return;
+    const int64_t seg = Q.tail_owner[j];
+    if (seg < 0) return;
+    const int t = Q.chunks[j].table;
+    const TableDev& td = P.tables[t];
+    const int64_t e = O.seg_start[seg + 1];
+    const int64_t m = pieces_after(Q, j, e, total);
+    float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
+    combine_pieces(Q, j, m, td.dim, P.dmax, lane, [&](int x0, double (&acc)[4]) {
+        *reinterpret_cast<float4*>(dst + x0) =
+            make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                        static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+    });
 }
 
 // ---------------------------------------------------------------- launchers
@@ -407,7 +403,9 @@ void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const f
 
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s) {
-    bwd_fixup_kernel<<<warp_grid(chunk_bound, num_sms * 8), kWarpThreads, 0, s>>>(P, Q, O);
+    (void)num_sms;  // one warp per chunk
+    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
+    bwd_fixup_kernel<<<static_cast<unsigned>(max64(need, 1)), kWarpThreads, 0, s>>>(P, Q, O);
 }
 
 }  // namespace cbtbe

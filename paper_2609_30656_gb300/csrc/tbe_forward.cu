@@ -114,40 +114,30 @@ __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
 }
 
 // A bag split over chunks: its tail piece (chunk where it starts) plus the head
-// pieces of the following chunks, added in chunk order in fp64, then scaled.
-__global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(Problem P, Plan Q, float* out) {
+// pieces of the following chunks, added in fp64, then scaled. One warp per chunk.
+__global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(const __grid_constant__ Problem P,
+                                                                 const __grid_constant__ Plan Q,
+                                                                 float* out) {
     const int lane = threadIdx.x & 31;
-    const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
-    for (int64_t j = warp_id_global(); j < total; j += warps_in_grid()) {
-        const int64_t bag = Q.tail_owner[j];
-        if (bag < 0) continue;
-        const int t = Q.chunks[j].table;
-        const TableDev& td = P.tables[t];
-        const int64_t s = load_index(P.offsets, bag, P.is32);
-        const int64_t e = load_index(P.offsets, bag + 1, P.is32);
-        float* dst = out + (bag - static_cast<int64_t>(t) * P.B) * P.sum_d + td.doff;
-        for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
-            const float4 a = *reinterpret_cast<const float4*>(Q.carry_tail + j * P.dmax + x0);
-            double acc[4] = {a.x, a.y, a.z, a.w};
-            for (int64_t jj = j + 1; jj < total; ++jj) {
-                const Chunk c2 = Q.chunks[jj];
-                if (c2.table != t || c2.first != bag || c2.k0 >= e) break;
-                const float4 h = *reinterpret_cast<const float4*>(Q.carry_head + jj * P.dmax + x0);
-                acc[0] += h.x;
-                acc[1] += h.y;
-                acc[2] += h.z;
-                acc[3] += h.w;
-                if (e <= c2.k0 + static_cast<int64_t>(c2.len & 0x7fffffffu)) break;
-            }
-            if (P.mean && e > s) {
-                const double L = static_cast<double>(e - s);
-                for (int x = 0; x < 4; ++x) acc[x] /= L;
-            }
-            *reinterpret_cast<float4*>(dst + x0) =
-                make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
-                            static_cast<float>(acc[2]), static_cast<float>(acc[3]));
-        }
-    }
+    const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    const int64_t j = warp_id_global();
+    if (j >= total) return;
+    const int64_t bag = Q.tail_owner[j];
+    if (bag < 0) return;
+    const int t = Q.chunks[j].table;
+    const TableDev& td = P.tables[t];
+    const int64_t s = load_index(P.offsets, bag, P.is32);
+    const int64_t e = load_index(P.offsets, bag + 1, P.is32);
+    const int64_t m = pieces_after(Q, j, e, total);
+    const double L = (P.mean && e > s) ? static_cast<double>(e - s) : 0.0;
+    float* dst = out + (bag - static_cast<int64_t>(t) * P.B) * P.sum_d + td.doff;
+    combine_pieces(Q, j, m, td.dim, P.dmax, lane, [&](int x0, double (&acc)[4]) {
+        if (L > 0.0)
+            for (int x = 0; x < 4; ++x) acc[x] /= L;
+        *reinterpret_cast<float4*>(dst + x0) =
+            make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                        static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+    });
 }
 
 template <int DT, int VPL, bool W>
@@ -190,9 +180,9 @@ void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int
 
 void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
                       int num_sms, cudaStream_t s) {
+    (void)num_sms;  // one warp per chunk
     const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
-    const int grid = static_cast<int>(min64(need, static_cast<int64_t>(num_sms) * 8));
-    fwd_fixup_kernel<<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out);
+    fwd_fixup_kernel<<<static_cast<unsigned>(max64(need, 1)), kWarpThreads, 0, s>>>(P, Q, out);
 }
 
 }  // namespace cbtbe

@@ -400,6 +400,70 @@ __device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const ui
     }
 }
 
+// ---------------------------------------------------------------- fix-up
+
+// A segment that straddles chunks left its tail piece in chunk j and head pieces
+// in the m chunks after it (chunks of a table are contiguous and chunk_len long
+// except the table's last, so m follows from the segment end). The pieces are
+// added in fp64 in a fixed order, so the result is deterministic; `store`
+// receives each group of four columns. Few pieces: lanes own columns and walk
+// the pieces; many pieces (a hot row repeated across hundreds of chunks): lanes
+// own pieces and meet in a butterfly per group of four columns.
+template <class Store>
+__device__ __forceinline__ void combine_pieces(const Plan& Q, int64_t j, int64_t m, int dim,
+                                               int dmax, int lane, Store store) {
+    const float* tail = Q.carry_tail + j * dmax;
+    const float* head = Q.carry_head + (j + 1) * dmax;
+    if (m <= 16) {
+        for (int x0 = lane * 4; x0 < dim; x0 += 128) {
+            const float4 a = *reinterpret_cast<const float4*>(tail + x0);
+            double acc[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll 4
+            for (int64_t i = 0; i < m; ++i) {
+                const float4 h = *reinterpret_cast<const float4*>(head + i * dmax + x0);
+                acc[0] += h.x;
+                acc[1] += h.y;
+                acc[2] += h.z;
+                acc[3] += h.w;
+            }
+            store(x0, acc);
+        }
+        return;
+    }
+    for (int x0 = 0; x0 < dim; x0 += 4) {
+        double acc[4] = {0.0, 0.0, 0.0, 0.0};
+        if (lane == 0) {
+            const float4 a = *reinterpret_cast<const float4*>(tail + x0);
+            acc[0] = a.x;
+            acc[1] = a.y;
+            acc[2] = a.z;
+            acc[3] = a.w;
+        }
+#pragma unroll 4
+        for (int64_t i = lane; i < m; i += 32) {
+            const float4 h = *reinterpret_cast<const float4*>(head + i * dmax + x0);
+            acc[0] += h.x;
+            acc[1] += h.y;
+            acc[2] += h.z;
+            acc[3] += h.w;
+        }
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1)
+#pragma unroll
+            for (int x = 0; x < 4; ++x) acc[x] += __shfl_xor_sync(kFull, acc[x], off);
+        if (lane == 0) store(x0, acc);
+    }
+}
+
+// Number of chunks after chunk j that a segment ending at `e` reaches into.
+__device__ __forceinline__ int64_t pieces_after(const Plan& Q, int64_t j, int64_t e, int64_t total) {
+    const Chunk ch = Q.chunks[j];
+    const int64_t k1 = ch.k0 + static_cast<int64_t>(ch.len & 0x7fffffffu);
+    if (e <= k1) return 0;
+    const int64_t m = (e - k1 + Q.chunk_len - 1) / Q.chunk_len;
+    return min64(m, total - j - 1);
+}
+
 // ---------------------------------------------------------------- small scans
 
 // Inclusive warp scan.
