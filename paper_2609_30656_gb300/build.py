@@ -19,8 +19,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcb_tbe.so")
-SOURCES = ["cb_tbe.cu", "tbe_plan.cu", "tbe_forward.cu", "tbe_backward.cu", "tbe_sort.cu",
-           "cb_tbe_noalloc.cu"]
+SOURCES = ["cb_tbe.cu", "tbe_plan.cu", "tbe_forward.cu", "tbe_forward_f32.cu", "tbe_forward_f16.cu",
+           "tbe_forward_bf16.cu", "tbe_backward.cu", "tbe_sort.cu", "cb_tbe_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -25,6 +25,7 @@ const char* const kComponentNames[kNumTimers] = {"fwd.prep",   "fwd.gather", "fw
 struct KernelClass {
     int dtype;  // storage dtype (forward) or CB_F32 (backward)
     int vpl;    // 16-byte vectors per lane: 1, 2 or 4
+    int gc;     // rows per warp step fixed at compile time (0: run time)
     std::vector<int32_t> tables;
 };
 
@@ -321,17 +322,19 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     for (int32_t t = 0; t < num_tables; ++t) {
         TableDev& td = h->tables[t];
         const int fv = vpl_for(td.row_vecs), bv = vpl_for(td.grad_vecs);
-        auto put = [&](std::vector<KernelClass>& cls, int dt, int v) {
+        const int fg = compile_time_groups(fv, td.lanes, td.groups);
+        const int bg = compile_time_groups(bv, td.grad_lanes, td.grad_groups);
+        auto put = [&](std::vector<KernelClass>& cls, int dt, int v, int gc) {
             for (size_t c = 0; c < cls.size(); ++c)
-                if (cls[c].dtype == dt && cls[c].vpl == v) {
+                if (cls[c].dtype == dt && cls[c].vpl == v && cls[c].gc == gc) {
                     cls[c].tables.push_back(t);
                     return static_cast<int>(c);
                 }
-            cls.push_back({dt, v, {t}});
+            cls.push_back({dt, v, gc, {t}});
             return static_cast<int>(cls.size() - 1);
         };
-        td.fwd_class = put(h->fwd_classes, td.dtype, fv);
-        td.bwd_class = put(h->bwd_classes, CB_F32, bv);
+        td.fwd_class = put(h->fwd_classes, td.dtype, fv, fg);
+        td.bwd_class = put(h->bwd_classes, CB_F32, bv, bg);
     }
 
     if (cudaGetDevice(&h->device) != cudaSuccess ||
@@ -436,7 +439,7 @@ cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t 
     record(h, h->ev_fwd[1], stream);
     for (size_t c = 0; c < h->fwd_classes.size(); ++c) {
         launch_fwd_gather(P, Q, out, static_cast<int>(c), h->fwd_classes[c].dtype,
-                          h->fwd_classes[c].vpl, bound, h->num_sms, stream);
+                          h->fwd_classes[c].vpl, h->fwd_classes[c].gc, bound, h->num_sms, stream);
         h->launches += 1;
     }
     record(h, h->ev_fwd[2], stream);
@@ -555,8 +558,8 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
     // (5) segmented reduce, (6) fix-up of runs split across chunks
     if (g->grads) {
         for (size_t c = 0; c < h->bwd_classes.size(); ++c) {
-            launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl, packed,
-                              bound, h->num_sms, stream);
+            launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl,
+                              h->bwd_classes[c].gc, packed, bound, h->num_sms, stream);
             h->launches += 1;
         }
         launch_bwd_fixup(P, Q, O, bound, h->num_sms, stream);

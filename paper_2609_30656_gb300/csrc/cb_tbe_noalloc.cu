@@ -82,7 +82,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
 
     // Table descriptors and kernel classes, exactly as cb_tbe_create builds them.
     std::vector<TableDev> td(num_tables);
-    struct Cls { int dtype, vpl; std::vector<int32_t> t; };
+    struct Cls { int dtype, vpl, gc; std::vector<int32_t> t; };
     std::vector<Cls> classes;
     int64_t row_base = 0, doff = 0;
     int32_t dmax = 0;
@@ -107,11 +107,13 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
         x.grad_vecs = d.dim / 4;
         split(x.grad_vecs, &x.grad_lanes, &x.grad_groups);
         const int vpl = x.row_vecs <= 32 ? 1 : (x.row_vecs <= 64 ? 2 : 4);
+        const int gc = compile_time_groups(vpl, x.lanes, x.groups);
         int c = -1;
         for (size_t k = 0; k < classes.size(); ++k)
-            if (classes[k].dtype == d.dtype && classes[k].vpl == vpl) c = static_cast<int>(k);
+            if (classes[k].dtype == d.dtype && classes[k].vpl == vpl && classes[k].gc == gc)
+                c = static_cast<int>(k);
         if (c < 0) {
-            classes.push_back({d.dtype, vpl, {}});
+            classes.push_back({d.dtype, vpl, gc, {}});
             c = static_cast<int>(classes.size() - 1);
         }
         classes[c].t.push_back(t);
@@ -209,7 +211,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
         launch_plan(P, Q, 0, nullptr, nullptr, num_sms, true, stream);
         for (size_t c = 0; c < classes.size(); ++c)
             launch_fwd_gather(P, Q, out, static_cast<int>(c), classes[c].dtype, classes[c].vpl,
-                              max_chunks, num_sms, stream);
+                              classes[c].gc, max_chunks, num_sms, stream);
         launch_fwd_fixup(P, Q, out, max_chunks, num_sms, stream);
     }
     if (cudaGetLastError() != cudaSuccess) return CB_ERR_CUDA;

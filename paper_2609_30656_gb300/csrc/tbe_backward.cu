@@ -281,7 +281,7 @@ struct BwdPolicy {
     }
 };
 
-template <int VPL, bool PACKED>
+template <int VPL, bool PACKED, int GC>
 __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
     bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
                       const __grid_constant__ BwdOut O, const float* grad_out, int cls) {
@@ -311,7 +311,7 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
         c.row_vecs = td.grad_vecs;
         c.last = false;
         if (lane == 0) Q.tail_owner[j] = -1;
-        walk_chunk(pol, c, P.zero_row, lane);
+        walk_chunk<BwdPolicy<VPL, PACKED>, GC>(pol, c, P.zero_row, lane);
     }
 }
 
@@ -381,23 +381,25 @@ void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s) {
     bwd_finalize_kernel<<<1, 1024, 0, s>>>(P, O);
 }
 
-template <int VPL, bool PACKED>
+template <int VPL, bool PACKED, int GC>
 static void launch_reduce_one(const Problem& P, const Plan& Q, const BwdOut& O, const float* go,
                               int cls, int64_t chunk_bound, int num_sms, cudaStream_t s) {
-    static int cap = occupancy_grid(bwd_reduce_kernel<VPL, PACKED>, kWarpThreads, num_sms);
-    bwd_reduce_kernel<VPL, PACKED><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, O, go, cls);
+    static int cap = occupancy_grid(bwd_reduce_kernel<VPL, PACKED, GC>, kWarpThreads, num_sms);
+    bwd_reduce_kernel<VPL, PACKED, GC><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, O, go, cls);
 }
 
 void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
-                       int cls, int vpl, bool packed, int64_t chunk_bound, int num_sms,
+                       int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
                        cudaStream_t s) {
-#define CB_CASE(V, PK)                                                              \
-    if (vpl == V && packed == PK) {                                                 \
-        launch_reduce_one<V, PK>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s); \
-        return;                                                                     \
+#define CB_CASE(V, G, PK)                                                                \
+    if (vpl == V && gc == G && packed == PK) {                                            \
+        launch_reduce_one<V, PK, G>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s);    \
+        return;                                                                          \
     }
-    CB_CASE(1, false) CB_CASE(2, false) CB_CASE(4, false)
-    CB_CASE(1, true) CB_CASE(2, true) CB_CASE(4, true)
+    CB_CASE(1, 1, false) CB_CASE(1, 2, false) CB_CASE(1, 4, false) CB_CASE(1, 8, false)
+    CB_CASE(1, 0, false) CB_CASE(2, 1, false) CB_CASE(4, 1, false)
+    CB_CASE(1, 1, true) CB_CASE(1, 2, true) CB_CASE(1, 4, true) CB_CASE(1, 8, true)
+    CB_CASE(1, 0, true) CB_CASE(2, 1, true) CB_CASE(4, 1, true)
 #undef CB_CASE
 }
 

@@ -1,117 +1,9 @@
-// tbe_forward.cu -- forward gather-pool of the pooled embedding bag
-// (sparse_arch lookups, Sec. IV.A.2; jagged categorical features, Abstract):
-//   out[b, Doff_t + j] = s_b * sum_{i in bag(t, b)} w_i * E_t[indices[i], j]
-//
-// One warp per chunk of lookup positions. A stored row is spread over V lanes
-// (16 bytes per lane per vector, V = row bytes / 16 up to 32), and a warp step
-// gathers G = 32 / V rows of the chunk at once, each lane keeping up to eight
-// 16-byte loads in flight. Rows widen to fp32 in registers; the G per-row
-// partial sums of a bag meet through warp shuffles when the bag is emitted.
+// tbe_forward.cu -- forward fix-up (bags split across chunks) and the launch
+// switch over storage types; the gather-pool kernel is in tbe_forward.cuh.
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
 
 namespace cbtbe {
-
-template <int DT, int VPL, bool WEIGHTED>
-struct FwdPolicy {
-    static constexpr int kDtype = DT;
-    static constexpr int kElems = Storage<DT>::kElems;
-    static constexpr int kVpl = VPL;
-    static constexpr int kUnroll = CB_WALK_ROWS / VPL > 0 ? CB_WALK_ROWS / VPL : 1;
-    static constexpr bool kWeighted = WEIGHTED;
-
-    const Problem& P;  // kernel parameters: read in place, not held in registers
-    const Plan& Q;
-    float* out;
-    const uint4* base;  // the table
-    int64_t rows;
-    uint32_t stride;    // 16-byte vectors per row
-    int32_t row_vecs;
-    int32_t chunk;
-    int32_t bag_lo;
-    int32_t doff;
-
-    __device__ __forceinline__ int64_t seg_begin(int32_t s) const { return load_index(P.offsets, s, P.is32); }
-    __device__ __forceinline__ int64_t seg_end(int32_t s) const { return load_index(P.offsets, s + 1, P.is32); }
-    struct Raw {
-        int64_t r;
-        float w;
-    };
-    __device__ __forceinline__ static Raw none() { return {-1, 0.f}; }
-    __device__ __forceinline__ Raw fetch(int64_t q) const {
-        return {load_index(P.indices, q, P.is32), WEIGHTED ? __ldg(P.weights + q) : 1.f};
-    }
-    // Row id of a lookup, checked once here; an out-of-range id contributes nothing.
-    __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
-        w = x.w;
-        if (x.r < 0 || x.r >= rows) {
-            set_error(P.error, CB_ERR_INDEX_OOB);
-            a = kInvalid;
-        } else {
-            a = static_cast<uint32_t>(x.r);
-        }
-    }
-    __device__ __forceinline__ void emit(int32_t bag, int32_t L, bool started, bool ends,
-                                         float (&tot)[VPL][kElems], int v, bool group0) const {
-        if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = bag;
-        if (!group0) return;
-        float* dst;
-        float scale = 0.f;
-        if (started && ends) {
-            dst = out + static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff;
-            if (P.mean && L > 0) scale = static_cast<float>(L);
-        } else {
-            dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
-        }
-        if (scale > 0.f) {  // mean pooling of a complete, non-empty bag
-#pragma unroll
-            for (int k = 0; k < VPL; ++k)
-#pragma unroll
-                for (int x = 0; x < kElems; ++x) tot[k][x] = tot[k][x] / scale;
-        }
-#pragma unroll
-        for (int k = 0; k < VPL; ++k) {
-            const int vec = v + 32 * k;
-            if (vec >= row_vecs) continue;
-            float4* d4 = reinterpret_cast<float4*>(dst + vec * kElems);
-#pragma unroll
-            for (int x = 0; x < kElems / 4; ++x)
-                d4[x] = make_float4(tot[k][4 * x], tot[k][4 * x + 1], tot[k][4 * x + 2], tot[k][4 * x + 3]);
-        }
-    }
-};
-
-template <int DT, int VPL, bool WEIGHTED>
-__global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
-    fwd_gather_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q, float* out,
-                      int cls) {
-    const int lane = threadIdx.x & 31;
-    const int64_t cb = Q.class_chunk_base[cls];
-    const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
-    for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
-        const Chunk ch = Q.chunks[j];
-        const TableDev& td = P.tables[ch.table];
-        FwdPolicy<DT, VPL, WEIGHTED> pol{P, Q, out};
-        pol.base = static_cast<const uint4*>(td.data);
-        pol.rows = td.rows;
-        pol.stride = static_cast<uint32_t>(td.row_vecs);
-        pol.row_vecs = td.row_vecs;
-        pol.chunk = static_cast<int32_t>(j);
-        pol.bag_lo = ch.table * P.B;
-        pol.doff = td.doff;
-        ChunkCtx c;
-        c.k0 = ch.k0;
-        c.len = static_cast<int32_t>(ch.len & 0x7fffffffu);
-        c.first = static_cast<int32_t>(ch.first);
-        c.seg_hi = pol.bag_lo + P.B;
-        c.lanes = td.lanes;
-        c.groups = td.groups;
-        c.row_vecs = td.row_vecs;
-        c.last = (ch.len >> 31) != 0;
-        if (lane == 0) Q.tail_owner[j] = -1;
-        walk_chunk(pol, c, P.zero_row, lane);
-    }
-}
 
 // A bag split over chunks: its tail piece (chunk where it starts) plus the head
 // pieces of the following chunks, added in fp64, then scaled. One warp per chunk.
@@ -140,42 +32,18 @@ __global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(const __grid_co
     });
 }
 
-template <int DT, int VPL, bool W>
-static int gather_grid(int num_sms) {
-    static int per_sm = -1;
-    if (per_sm < 0) {
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fwd_gather_kernel<DT, VPL, W>,
-                                                          kWarpThreads, 0) != cudaSuccess ||
-            per_sm < 1)
-            per_sm = 1;
-    }
-    return per_sm * num_sms;
-}
-
-template <int DT, int VPL>
-static void launch_one(const Problem& P, const Plan& Q, float* out, int cls, int64_t chunk_bound,
-                       int num_sms, cudaStream_t s) {
-    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
-    if (P.weights) {
-        const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL, true>(num_sms)));
-        fwd_gather_kernel<DT, VPL, true><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
-    } else {
-        const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL, false>(num_sms)));
-        fwd_gather_kernel<DT, VPL, false><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
-    }
-}
+void launch_fwd_gather_f32(const Problem&, const Plan&, float*, int, int, int, int64_t, int,
+                           cudaStream_t);
+void launch_fwd_gather_f16(const Problem&, const Plan&, float*, int, int, int, int64_t, int,
+                           cudaStream_t);
+void launch_fwd_gather_bf16(const Problem&, const Plan&, float*, int, int, int, int64_t, int,
+                            cudaStream_t);
 
 void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,
-                       int64_t chunk_bound, int num_sms, cudaStream_t s) {
-#define CB_CASE(D, V)                                              \
-    if (dtype == D && vpl == V) {                                  \
-        launch_one<D, V>(P, Q, out, cls, chunk_bound, num_sms, s); \
-        return;                                                    \
-    }
-    CB_CASE(CB_F32, 1) CB_CASE(CB_F32, 2) CB_CASE(CB_F32, 4)
-    CB_CASE(CB_F16, 1) CB_CASE(CB_F16, 2) CB_CASE(CB_F16, 4)
-    CB_CASE(CB_BF16, 1) CB_CASE(CB_BF16, 2) CB_CASE(CB_BF16, 4)
-#undef CB_CASE
+                       int gc, int64_t chunk_bound, int num_sms, cudaStream_t s) {
+    if (dtype == CB_F32) launch_fwd_gather_f32(P, Q, out, cls, vpl, gc, chunk_bound, num_sms, s);
+    else if (dtype == CB_F16) launch_fwd_gather_f16(P, Q, out, cls, vpl, gc, chunk_bound, num_sms, s);
+    else launch_fwd_gather_bf16(P, Q, out, cls, vpl, gc, chunk_bound, num_sms, s);
 }
 
 void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,

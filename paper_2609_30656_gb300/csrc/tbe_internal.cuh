@@ -228,14 +228,19 @@ __device__ __forceinline__ int32_t rel_pos(int64_t x, int64_t k0) {
     return r < kRelLo ? kRelLo : (r > kRelHi ? kRelHi : static_cast<int32_t>(r));
 }
 
-template <class Pol>
+// GC > 0: the row layout is known at compile time (G = GC rows per warp step,
+// V = 32 / GC lanes per row); GC == 0: taken from the chunk at run time (rows
+// whose vector count is not a power of two).
+template <class Pol, int GC>
 __device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const uint4* zero_row,
                                            int lane) {
     constexpr int E = Pol::kElems;
     constexpr int VPL = Pol::kVpl;
     constexpr int U = Pol::kUnroll;
     constexpr bool W = Pol::kWeighted;
-    const int V = c.lanes, G = c.groups;
+    constexpr bool kExact = GC > 0 && VPL == 1;  // each lane owns one vector of one row
+    const int V = GC > 0 ? 32 / GC : c.lanes;
+    const int G = GC > 0 ? GC : c.groups;
     const int g = lane / V;
     const int v = lane - g * V;
     const int ustop = min(U, 32 / G);  // row groups per step
@@ -246,7 +251,7 @@ __device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const ui
     bool vlive[VPL];
 #pragma unroll
     for (int k = 0; k < VPL; ++k) {
-        vlive[k] = g < G && v + 32 * k < c.row_vecs;
+        vlive[k] = kExact || (g < G && v + 32 * k < c.row_vecs);
         vzero[k] = zero_row + (v + 32 * k) % 128;
     }
 
@@ -430,28 +435,44 @@ __device__ __forceinline__ void combine_pieces(const Plan& Q, int64_t j, int64_t
         }
         return;
     }
-    for (int x0 = 0; x0 < dim; x0 += 4) {
-        double acc[4] = {0.0, 0.0, 0.0, 0.0};
+    // Four groups of four columns per round: 16 independent loads per lane.
+    for (int x0 = 0; x0 < dim; x0 += 16) {
+        double acc[4][4] = {};
+        const int ng = min(4, (dim - x0) / 4);
         if (lane == 0) {
-            const float4 a = *reinterpret_cast<const float4*>(tail + x0);
-            acc[0] = a.x;
-            acc[1] = a.y;
-            acc[2] = a.z;
-            acc[3] = a.w;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (c >= ng) break;
+                const float4 a = *reinterpret_cast<const float4*>(tail + x0 + 4 * c);
+                acc[c][0] = a.x;
+                acc[c][1] = a.y;
+                acc[c][2] = a.z;
+                acc[c][3] = a.w;
+            }
         }
 #pragma unroll 4
         for (int64_t i = lane; i < m; i += 32) {
-            const float4 h = *reinterpret_cast<const float4*>(head + i * dmax + x0);
-            acc[0] += h.x;
-            acc[1] += h.y;
-            acc[2] += h.z;
-            acc[3] += h.w;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (c >= ng) break;
+                const float4 h = *reinterpret_cast<const float4*>(head + i * dmax + x0 + 4 * c);
+                acc[c][0] += h.x;
+                acc[c][1] += h.y;
+                acc[c][2] += h.z;
+                acc[c][3] += h.w;
+            }
         }
 #pragma unroll
         for (int off = 16; off >= 1; off >>= 1)
 #pragma unroll
-            for (int x = 0; x < 4; ++x) acc[x] += __shfl_xor_sync(kFull, acc[x], off);
-        if (lane == 0) store(x0, acc);
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int x = 0; x < 4; ++x) acc[c][x] += __shfl_xor_sync(kFull, acc[c][x], off);
+        if (lane == 0) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < ng) store(x0 + 4 * c, acc[c]);
+        }
     }
 }
 

@@ -60,7 +60,7 @@ void launch_plan(const Problem& P, const Plan& Q, int mode, const uint32_t* seg_
                  const int64_t* num_unique, int num_sms, bool tables_too, cudaStream_t s);
 
 void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,
-                       int64_t chunk_bound, int num_sms, cudaStream_t s);
+                       int gc, int64_t chunk_bound, int num_sms, cudaStream_t s);
 void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
 
@@ -75,8 +75,15 @@ void launch_rle(const uint32_t* keys, int64_t n, int64_t* tile_heads, int64_t* t
                 int64_t* num_unique, uint32_t* uniq, uint32_t* seg_start, cudaStream_t s);
 void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s);
 void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
-                       int cls, int vpl, bool packed, int64_t chunk_bound, int num_sms,
+                       int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
                        cudaStream_t s);
+// Rows per warp step fixed at compile time for a row of `vecs` 16-byte vectors
+// spread as (lanes, groups), or 0 when the layout is only known at run time.
+inline int compile_time_groups(int vpl, int lanes, int groups) {
+    if (vpl > 1) return 1;
+    if (lanes * groups == 32 && (groups == 1 || groups == 2 || groups == 4 || groups == 8)) return groups;
+    return 0;
+}
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
 
