@@ -107,17 +107,43 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
 
 // ---------------------------------------------------------------- (3) runs
 
-__device__ __forceinline__ bool is_head(const uint32_t* keys, int64_t i) {
-    return i == 0 || __ldg(keys + i) != __ldg(keys + i - 1);
+// Head flags of the kRleItems sorted keys starting at `base` (thread-blocked):
+// bit i is set when key[base + i] starts a run. Full groups load as four
+// 16-byte vectors; the key before the group comes from the previous lane.
+__device__ __forceinline__ uint32_t head_flags(const uint32_t* keys, int64_t n, int64_t base) {
+    uint32_t k[kRleItems];
+    if (base + kRleItems <= n) {
+        const uint4* v = reinterpret_cast<const uint4*>(keys + base);
+#pragma unroll
+        for (int i = 0; i < kRleItems / 4; ++i) {
+            const uint4 x = __ldg(v + i);
+            k[4 * i] = x.x;
+            k[4 * i + 1] = x.y;
+            k[4 * i + 2] = x.z;
+            k[4 * i + 3] = x.w;
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < kRleItems; ++i) k[i] = base + i < n ? __ldg(keys + base + i) : 0u;
+    }
+    const int lane = threadIdx.x & 31;
+    uint32_t prev = __shfl_up_sync(kFull, k[kRleItems - 1], 1);
+    if (lane == 0 && base > 0 && base <= n) prev = __ldg(keys + base - 1);
+    uint32_t flags = 0;
+#pragma unroll
+    for (int i = 0; i < kRleItems; ++i) {
+        const uint32_t before = i == 0 ? prev : k[i - 1];
+        const bool head = base + i < n && (base + i == 0 || k[i] != before);
+        flags |= head ? (1u << i) : 0u;
+    }
+    return flags;
 }
 
 __global__ void __launch_bounds__(kRleThreads) rle_count_kernel(const uint32_t* keys, int64_t n,
                                                                  int64_t* tile_heads) {
     __shared__ int64_t sh[33];
     const int64_t base = static_cast<int64_t>(blockIdx.x) * kRleTile + threadIdx.x * kRleItems;
-    int64_t c = 0;
-    for (int i = 0; i < kRleItems; ++i)
-        if (base + i < n && is_head(keys, base + i)) ++c;
+    const int64_t c = __popc(head_flags(keys, n, base));
     int64_t total;
     block_excl_scan(c, sh, &total);
     if (threadIdx.x == 0) tile_heads[blockIdx.x] = total;
@@ -148,21 +174,15 @@ __global__ void __launch_bounds__(kRleThreads) rle_write_kernel(const uint32_t* 
                                                                 uint32_t* uniq, uint32_t* seg_start) {
     __shared__ int64_t sh[33];
     const int64_t base = static_cast<int64_t>(blockIdx.x) * kRleTile + threadIdx.x * kRleItems;
-    uint32_t flags = 0;
-    int64_t c = 0;
-    for (int i = 0; i < kRleItems; ++i)
-        if (base + i < n && is_head(keys, base + i)) {
-            flags |= 1u << i;
-            ++c;
-        }
+    const uint32_t flags = head_flags(keys, n, base);
     int64_t total;
-    int64_t u = tile_base[blockIdx.x] + block_excl_scan(c, sh, &total);
-    for (int i = 0; i < kRleItems; ++i)
-        if (flags & (1u << i)) {
-            uniq[u] = __ldg(keys + base + i);
-            seg_start[u] = static_cast<uint32_t>(base + i);
-            ++u;
-        }
+    int64_t u = tile_base[blockIdx.x] + block_excl_scan(__popc(flags), sh, &total);
+    for (uint32_t f = flags; f; f &= f - 1) {
+        const int i = __ffs(f) - 1;
+        uniq[u] = __ldg(keys + base + i);
+        seg_start[u] = static_cast<uint32_t>(base + i);
+        ++u;
+    }
     if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) seg_start[*num_unique] = static_cast<uint32_t>(n);
 }
 

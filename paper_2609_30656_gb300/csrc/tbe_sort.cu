@@ -136,12 +136,25 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
             }
             k -= used;
             if (!done && used == 0) {
-                if ((++spins & 63u) == 0 && global_ns() - t0 > S.timeout_ns) {
+                // The nearest predecessor has not published yet: poll that one
+                // word alone, backing off, then read the window again.
+                const uint32_t* src = (S.force_timeout && tile == 1) ? S.never_set
+                                                                     : S.status + k * kRadix + d;
+                uint32_t ns = 32;
+                bool timed_out = false;
+                while ((load_volatile(src) & ~kCountMask) == 0) {
+                    if ((++spins & 15u) == 0 && global_ns() - t0 > S.timeout_ns) {
+                        timed_out = true;
+                        break;
+                    }
+                    __nanosleep(ns);
+                    ns = ns < 512 ? 2 * ns : ns;
+                }
+                if (timed_out) {
                     set_error(S.error, CB_ERR_TIMEOUT);
                     atomicExch(&sh_abort, 1);
                     break;
                 }
-                __nanosleep(32);
             }
         }
         store_volatile(my_status, kFlagIncl | ((excl + count) & kCountMask));
