@@ -59,6 +59,12 @@ struct Workspace {
     float* carry_tail = nullptr;
     int64_t* tail_owner = nullptr;
     int64_t max_chunks = 0;
+    // radix sort plan: table-aligned tiles
+    int64_t* sp_table_pos = nullptr;
+    int64_t* sp_ord = nullptr;
+    int64_t* sp_class_base = nullptr;
+    Chunk* sp_tiles = nullptr;
+    int64_t sp_max_tiles = 0;
     // backward
     uint32_t* keys[2] = {nullptr, nullptr};
     uint32_t* vals[2] = {nullptr, nullptr};
@@ -102,6 +108,8 @@ struct cb_tbe {
     int32_t* d_fwd_class_start = nullptr;
     int32_t* d_bwd_class_tables = nullptr;
     int32_t* d_bwd_class_start = nullptr;
+    int32_t* d_all_tables = nullptr;  // 0..T-1, one class: the radix sort plan
+    int32_t* d_all_start = nullptr;   // {0, T}
     int* d_error = nullptr;
     uint32_t* d_never_set = nullptr;
     uint4* d_zero_row = nullptr;  // 2 KB of zeros
@@ -145,13 +153,21 @@ size_t layout(const cb_tbe* h, int64_t B, int64_t n, char* base, Workspace* w) {
         ws.vals[i] = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
     }
     ws.packed = static_cast<uint2*>(take(sizeof(uint2) * n));
-    ws.hist = static_cast<uint32_t*>(take(sizeof(uint32_t) * 4 * 256));
-    ws.digit_base = static_cast<uint32_t*>(take(sizeof(uint32_t) * 4 * 256));
-    ws.sort_tiles = sort_num_tiles(n);
+    ws.sp_max_tiles = n / kSortTileKeys + T + 1;
+    ws.sp_table_pos = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.sp_ord = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.sp_class_base = static_cast<int64_t*>(take(sizeof(int64_t) * 2));
+    ws.sp_tiles = static_cast<Chunk*>(take(sizeof(Chunk) * ws.sp_max_tiles));
+    ws.sort_tiles = ws.sp_max_tiles;
+    const size_t hist_words = static_cast<size_t>(T) * h->passes * 256;
+    ws.digit_base = static_cast<uint32_t*>(take(sizeof(uint32_t) * hist_words));
     ws.status_bytes = sizeof(uint32_t) * static_cast<size_t>(h->passes) * ws.sort_tiles * 256;
-    // status and tile counters are adjacent so that one memset clears both
-    ws.status = static_cast<uint32_t*>(take(ws.status_bytes + sizeof(uint32_t) * 4));
+    // histograms, status words and tile counters are adjacent: one memset clears them
+    ws.hist = static_cast<uint32_t*>(take(sizeof(uint32_t) * hist_words + ws.status_bytes +
+                                          sizeof(uint32_t) * 4));
+    ws.status = base ? ws.hist + hist_words : nullptr;
     ws.tile_counters = base ? ws.status + static_cast<size_t>(h->passes) * ws.sort_tiles * 256 : nullptr;
+    ws.status_bytes += sizeof(uint32_t) * hist_words;  // bytes cleared from `hist` on
     const int64_t rt = rle_num_tiles(n);
     ws.tile_heads = static_cast<int64_t*>(take(sizeof(int64_t) * rt));
     ws.tile_base = static_cast<int64_t*>(take(sizeof(int64_t) * rt));
@@ -312,8 +328,11 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     }
     h->sum_rows = row_base;
     h->sum_d = static_cast<int32_t>(doff);
+    // Each table's range is sorted on its own, on the bits of the row number.
+    int64_t max_rows = 1;
+    for (const TableDev& td : h->tables) max_rows = std::max(max_rows, td.rows);
     int bits = 1;
-    while (bits < 32 && (int64_t(1) << bits) < row_base) ++bits;
+    while (bits < 32 && (int64_t(1) << bits) < max_rows) ++bits;
     h->key_bits = bits;
     h->passes = (bits + 7) / 8;
 
@@ -359,6 +378,10 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     const size_t o_fcs = off; off += align_up(sizeof(int32_t) * fcs.size());
     const size_t o_bct = off; off += align_up(sizeof(int32_t) * bct.size());
     const size_t o_bcs = off; off += align_up(sizeof(int32_t) * bcs.size());
+    std::vector<int32_t> all(num_tables), all_start{0, num_tables};
+    for (int32_t t = 0; t < num_tables; ++t) all[t] = t;
+    const size_t o_all = off; off += align_up(sizeof(int32_t) * num_tables);
+    const size_t o_alls = off; off += align_up(sizeof(int32_t) * 2);
     const size_t o_err = off; off += align_up(sizeof(int) + sizeof(uint32_t));
     const size_t o_zero = off; off += align_up(2048);
     if (cudaMalloc(&h->persist, off) != cudaSuccess) {
@@ -372,6 +395,8 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     h->d_fwd_class_start = reinterpret_cast<int32_t*>(p + o_fcs);
     h->d_bwd_class_tables = reinterpret_cast<int32_t*>(p + o_bct);
     h->d_bwd_class_start = reinterpret_cast<int32_t*>(p + o_bcs);
+    h->d_all_tables = reinterpret_cast<int32_t*>(p + o_all);
+    h->d_all_start = reinterpret_cast<int32_t*>(p + o_alls);
     h->d_error = reinterpret_cast<int*>(p + o_err);
     h->d_never_set = reinterpret_cast<uint32_t*>(p + o_err + sizeof(int));
     h->d_zero_row = reinterpret_cast<uint4*>(p + o_zero);
@@ -384,6 +409,10 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     ok = ok && cudaMemcpy(h->d_bwd_class_tables, bct.data(), sizeof(int32_t) * bct.size(),
                           cudaMemcpyHostToDevice) == cudaSuccess;
     ok = ok && cudaMemcpy(h->d_bwd_class_start, bcs.data(), sizeof(int32_t) * bcs.size(),
+                          cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemcpy(h->d_all_tables, all.data(), sizeof(int32_t) * num_tables,
+                          cudaMemcpyHostToDevice) == cudaSuccess;
+    ok = ok && cudaMemcpy(h->d_all_start, all_start.data(), sizeof(int32_t) * 2,
                           cudaMemcpyHostToDevice) == cudaSuccess;
     ok = ok && cudaMemset(h->d_error, 0, sizeof(int) + sizeof(uint32_t)) == cudaSuccess;
     ok = ok && cudaMemset(h->d_zero_row, 0, 2048) == cudaSuccess;
@@ -488,25 +517,37 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
     const int64_t bound = n / kBwdChunk + h->T + 1;
     const bool packed = per_sample_weights != nullptr || h->mode == CB_POOL_MEAN;
 
-    // (1) keys and digit histograms
+    // (1) keys and payloads
     launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
     h->launches += 2;
-    if (cudaMemsetAsync(w.hist, 0, sizeof(uint32_t) * 4 * 256, stream) != cudaSuccess ||
-        cudaMemsetAsync(w.status, 0, w.status_bytes + sizeof(uint32_t) * 4, stream) != cudaSuccess)
+    if (cudaMemsetAsync(w.hist, 0, w.status_bytes + sizeof(uint32_t) * 4, stream) != cudaSuccess)
         return CB_ERR_CUDA;
     KeyGen K;
     K.keys = w.keys[0];
     K.vals = w.vals[0];
     K.packed = packed ? w.packed : nullptr;
-    K.hist = w.hist;
-    K.passes = h->passes;
     launch_keygen(P, Q, K, packed, bound, h->num_sms, stream);
     h->launches += 1;
     record(h, h->ev_bwd[1], stream);
 
-    // (2) radix sort, 8 bits per pass
-    launch_digit_scan(w.hist, w.digit_base, h->passes, stream);
-    h->launches += 1;
+    // (2) radix sort of each table's range, 8 bits of the row number per pass
+    Plan SQ;
+    SQ.chunk_len = static_cast<int32_t>(kSortTileKeys);
+    SQ.num_classes = 1;
+    SQ.class_tables = h->d_all_tables;
+    SQ.class_table_start = h->d_all_start;
+    SQ.table_pos = w.sp_table_pos;
+    SQ.ord_chunk_base = w.sp_ord;
+    SQ.class_chunk_base = w.sp_class_base;
+    SQ.chunks = w.sp_tiles;
+    SQ.max_chunks = w.sp_max_tiles;
+    SQ.carry_head = SQ.carry_tail = nullptr;
+    SQ.tail_owner = nullptr;
+    launch_plan(P, SQ, 2, nullptr, nullptr, h->num_sms, true, stream);
+    launch_sort_hist(w.keys[0], w.sp_tiles, w.sp_class_base + 1, w.sp_max_tiles, h->d_tables,
+                     h->passes, w.hist, h->num_sms, stream);
+    launch_sort_bases(w.hist, w.sp_table_pos, h->T, h->passes, w.digit_base, stream);
+    h->launches += 4;
     int cur = 0;
     for (int p = 0; p < h->passes; ++p) {
         SortPass S;
@@ -514,16 +555,21 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
         S.vals_in = w.vals[cur];
         S.keys_out = w.keys[cur ^ 1];
         S.vals_out = w.vals[cur ^ 1];
+        S.tiles = w.sp_tiles;
+        S.num_tiles = w.sp_class_base + 1;
+        S.table_first_tile = w.sp_ord;
+        S.tables = h->d_tables;
         S.n = n;
         S.shift = 8 * p;
         S.digit_base = w.digit_base + 256 * p;
+        S.base_stride = 256 * h->passes;
         S.status = w.status + static_cast<size_t>(p) * w.sort_tiles * 256;
         S.tile_counter = w.tile_counters + p;
         S.never_set = h->d_never_set;
         S.force_timeout = (h->flags & CB_DEBUG_FORCE_LOOKBACK_TIMEOUT) && p == 0;
         S.error = h->d_error;
         S.timeout_ns = kLookbackTimeoutNs;
-        launch_onesweep(S, stream);
+        launch_onesweep(S, w.sp_max_tiles, stream);
         h->launches += 1;
         cur ^= 1;
     }

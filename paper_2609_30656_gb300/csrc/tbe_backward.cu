@@ -5,7 +5,7 @@
 // Steps: (1) key generation: one warp per chunk of lookups walks the bags and
 // writes key_i = row_base_t + indices[i] with a payload (the bag id, or the
 // lookup position plus a packed (bag, w_i * s_b) pair when a coefficient is
-// needed), counting the radix digit histograms on the way; (2) radix sort;
+// needed); (2) radix sort of each table's range;
 // (3) run-length pass over the sorted ids; (4) per-table unique ranges and
 // packed gradient offsets; (5) segmented reduce of the gathered grad_out
 // slices, one warp per chunk of sorted positions; (6) fp64 fix-up of runs that
@@ -23,9 +23,6 @@ constexpr int kRleTile = kRleThreads * kRleItems;
 
 template <bool PACKED>
 __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q, KeyGen K) {
-    __shared__ uint32_t sh_hist[4 * 256];
-    for (int i = threadIdx.x; i < 4 * 256; i += blockDim.x) sh_hist[i] = 0;
-    __syncthreads();
     const int lane = threadIdx.x & 31;
     const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     for (int64_t j = warp_id_global(); j < total; j += warps_in_grid()) {
@@ -83,26 +80,8 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
                     K.vals[q] = static_cast<uint32_t>(my_bag);
                 }
             }
-            // Digit histograms of every pass (warp-aggregated shared atomics).
-            // Digits that all lanes share (the high digits, inside one table)
-            // cost one shared atomic; the others one atomic per lane.
-            const uint32_t vmask = __ballot_sync(kFull, valid);
-            const uint32_t key = valid ? K.keys[q] : 0u;
-            const int leader = __ffs(vmask) - 1;
-            for (int p = 0; p < K.passes; ++p) {
-                const uint32_t dgt = (key >> (8 * p)) & 255u;
-                const uint32_t d0 = __shfl_sync(kFull, dgt, leader);
-                if (__all_sync(kFull, !valid || dgt == d0)) {
-                    if (lane == leader) atomicAdd(&sh_hist[p * 256 + d0], __popc(vmask));
-                } else if (valid) {
-                    atomicAdd(&sh_hist[p * 256 + dgt], 1u);
-                }
-            }
         }
     }
-    __syncthreads();
-    for (int i = threadIdx.x; i < K.passes * 256; i += blockDim.x)
-        if (sh_hist[i]) atomicAdd(K.hist + i, sh_hist[i]);
 }
 
 // ---------------------------------------------------------------- (3) runs

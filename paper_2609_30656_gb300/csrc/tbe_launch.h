@@ -9,15 +9,21 @@ namespace cbtbe {
 struct Problem;
 struct Plan;
 
-// One radix pass over n (key, payload) pairs.
+// One radix pass over n (key, payload) pairs, each table's range sorted on
+// its own: tiles never straddle tables, digits are taken from key - row_base_t.
 struct SortPass {
     const uint32_t* keys_in;
     const uint32_t* vals_in;
     uint32_t* keys_out;
     uint32_t* vals_out;
+    const struct Chunk* tiles;        // table-aligned tiles of at most 4096 positions
+    const int64_t* num_tiles;         // device scalar
+    const int64_t* table_first_tile;  // [T]
+    const struct TableDev* tables;
     int64_t n;
-    int shift;                   // digit = (key >> shift) & 255
-    const uint32_t* digit_base;  // [256] first output slot of each digit
+    int shift;                   // digit = ((key - row_base_t) >> shift) & 255
+    const uint32_t* digit_base;  // [T][stride]: this pass's 256 first output slots per table
+    int base_stride;             // passes * 256
     uint32_t* status;            // [tiles * 256], zeroed before the pass
     uint32_t* tile_counter;      // zeroed before the pass
     const uint32_t* never_set;   // a zero word no kernel writes (timeout test hook)
@@ -30,8 +36,6 @@ struct KeyGen {
     uint32_t* keys;    // [n] row_base_t + index
     uint32_t* vals;    // [n] bag id, or lookup position when `packed` is used
     uint2* packed;     // [n] (bag id, bits of w_i * s_b) by lookup position, or null
-    uint32_t* hist;    // [passes * 256], zeroed before
-    int passes;
 };
 
 struct BwdOut {
@@ -64,9 +68,13 @@ void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int
 void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
 
-int64_t sort_num_tiles(int64_t n);
-void launch_digit_scan(const uint32_t* hist, uint32_t* base, int passes, cudaStream_t s);
-void launch_onesweep(const SortPass& S, cudaStream_t s);
+constexpr int64_t kSortTileKeys = 4096;
+void launch_sort_hist(const uint32_t* keys, const struct Chunk* tiles, const int64_t* num_tiles,
+                      int64_t tile_bound, const struct TableDev* tables, int passes, uint32_t* hist,
+                      int num_sms, cudaStream_t s);
+void launch_sort_bases(const uint32_t* hist, const int64_t* table_pos, int T, int passes,
+                       uint32_t* base, cudaStream_t s);
+void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s);
 
 void launch_keygen(const Problem& P, const Plan& Q, const KeyGen& K, bool packed, int64_t chunk_bound,
                    int num_sms, cudaStream_t s);

@@ -65,6 +65,7 @@ __global__ void __launch_bounds__(1024) plan_tables_kernel(Problem P, Plan Q) {
 
 // mode 0: first = the bag touching the chunk start (forward, key generation).
 // mode 1: first = the run of sorted ids containing the chunk start (reduce).
+// mode 2: tiles only (radix sort), first left at 0.
 __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* seg_start,
                                    const int64_t* num_unique) {
     const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
@@ -87,8 +88,10 @@ __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* 
         const int64_t k0 = min(p0 + local * C, p1);
         const int64_t len = min(C, p1 - k0);
         const bool last = local >= nch - 1;
-        int64_t first;
-        if (mode == 0) {
+        int64_t first = 0;
+        if (mode == 2) {
+            // tiles only (radix sort): no first segment needed
+        } else if (mode == 0) {
             // First bag b of table t with offsets[b] >= k0 (lower bound over the
             // table's B + 1 offsets); the chunk starts in the bag before it unless
             // a bag starts exactly at k0.

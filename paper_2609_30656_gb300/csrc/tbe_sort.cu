@@ -1,14 +1,17 @@
 // tbe_sort.cu -- stable LSD radix sort of (row id, payload) pairs for the
 // de-duplicated backward of the pooled embedding bag.
 //
-// One pass per 8-bit digit. The digit histograms of every pass are counted once,
-// while the keys are generated; each pass then reads and writes every pair
-// exactly once ("onesweep"): a block takes the next tile id from a counter,
-// ranks its 4096 keys by digit (warp match + per-warp counters, stable by
-// position), publishes its per-digit counts, and finds the counts of all earlier
-// tiles by a decoupled look-back over their published words. The look-back wait
-// is bounded in time: when it runs out the kernel records CB_ERR_TIMEOUT,
-// publishes anyway so later tiles finish, and writes nothing.
+// A table's lookups are contiguous and its row ids are row_base_t + r with
+// r < rows_t, so each table's range is sorted on its own, on the bits of r only
+// (3 passes of 8 bits for tables of up to 16M rows). One streaming kernel counts
+// every pass's digit histogram per table; each pass then reads and writes every
+// pair exactly once ("onesweep"): a block takes the next tile (at most 4096
+// positions of one table) from a counter, ranks its keys by digit (warp match +
+// per-warp counters, stable by position), publishes its per-digit counts, and
+// finds the counts of the table's earlier tiles by a decoupled look-back over
+// their published words. The look-back wait is bounded in time: when it runs
+// out the kernel records CB_ERR_TIMEOUT, publishes anyway so later tiles
+// finish, and writes nothing.
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
 
@@ -17,6 +20,7 @@ namespace cbtbe {
 constexpr int kSortThreads = 256;
 constexpr int kSortItems = 16;
 constexpr int kSortTile = kSortThreads * kSortItems;  // 4096 keys
+static_assert(kSortTile == kSortTileKeys, "tile size shared with the host plan");
 constexpr int kRadix = 256;
 constexpr int kSortWarps = kSortThreads / 32;
 constexpr uint32_t kFlagAgg = 1u << 30;
@@ -58,8 +62,13 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     for (int i = tid; i < kSortWarps * kRadix; i += kSortThreads) (&sh_warp[0][0])[i] = 0;
     __syncthreads();
     const uint32_t tile = sh_tile;
-    const int64_t tile_base = static_cast<int64_t>(tile) * kSortTile;
-    const int tile_count = static_cast<int>(min64(kSortTile, S.n - tile_base));
+    if (tile >= *S.num_tiles) return;  // the grid is an upper bound on the tiles
+    const Chunk tc = S.tiles[tile];
+    const int t = tc.table;
+    const int64_t tile_base = tc.k0;
+    const int tile_count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tile_base));
+    const uint32_t row_base = static_cast<uint32_t>(S.tables[t].row_base);
+    const int64_t first_tile = S.table_first_tile[t];
 
     // Warp-striped load: item j of lane l is position tile_base + wid*512 + j*32 + l.
     // Payloads wait in shared memory; keys and ranks stay in registers.
@@ -78,7 +87,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         const bool valid = local < tile_count;
         const uint32_t vmask = __ballot_sync(kFull, valid);
-        const uint32_t d = (key[j] >> S.shift) & (kRadix - 1);
+        const uint32_t d = ((key[j] - row_base) >> S.shift) & (kRadix - 1);
         uint32_t peers = 0, before = 0, r = 0;
         if (valid) {
             peers = __match_any_sync(vmask, d);
@@ -102,7 +111,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         count += c;
     }
     uint32_t* my_status = S.status + static_cast<int64_t>(tile) * kRadix + d;
-    store_volatile(my_status, (tile == 0 ? kFlagIncl : kFlagAgg) | count);
+    store_volatile(my_status, (tile == first_tile ? kFlagIncl : kFlagAgg) | count);
     int64_t total;
     const int64_t start = block_excl_scan(count, sh_scan, &total);
     sh_start[d] = static_cast<uint32_t>(start);
@@ -110,7 +119,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     // Decoupled look-back over earlier tiles for digit d, kLookbackWindow
     // predecessors per round (independent loads), bounded in time.
     uint32_t excl = 0;
-    if (tile > 0) {
+    if (tile > first_tile) {
         int64_t k = static_cast<int64_t>(tile) - 1;
         const uint64_t t0 = global_ns();
         uint32_t spins = 0;
@@ -122,7 +131,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
                 const int64_t kk = k - w;
                 const uint32_t* src = (S.force_timeout && tile == 1) ? S.never_set
                                                                       : S.status + kk * kRadix + d;
-                word[w] = kk >= 0 ? load_volatile(src) : kFlagIncl;
+                word[w] = kk >= first_tile ? load_volatile(src) : kFlagIncl;
             }
             int used = 0;
 #pragma unroll
@@ -132,7 +141,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
                 if (flag == 0) continue;             // not published yet: poll it again
                 excl += word[w] & kCountMask;
                 used = w + 1;
-                if (flag == kFlagIncl || k - w == 0) done = true;
+                if (flag == kFlagIncl || k - w <= first_tile) done = true;
             }
             k -= used;
             if (!done && used == 0) {
@@ -159,7 +168,8 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         }
         store_volatile(my_status, kFlagIncl | ((excl + count) & kCountMask));
     }
-    sh_goff[d] = static_cast<long long>(S.digit_base[d]) + excl - static_cast<long long>(start);
+    sh_goff[d] = static_cast<long long>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) +
+                 excl - static_cast<long long>(start);
     __syncthreads();
 
     // Scatter into shared memory in tile-sorted order.
@@ -167,7 +177,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         if (local < tile_count) {
-            const uint32_t dd = (key[j] >> S.shift) & (kRadix - 1);
+            const uint32_t dd = ((key[j] - row_base) >> S.shift) & (kRadix - 1);
             const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
             const uint32_t pos = sh_start[dd] + sh_warp[wid][dd] + r;
             sh_keys[pos] = key[j];
@@ -179,7 +189,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     // Consecutive shared slots of one digit go to consecutive global slots.
     for (int i = tid; i < tile_count; i += kSortThreads) {
         const uint32_t k2 = sh_keys[i];
-        const long long dest = sh_goff[(k2 >> S.shift) & (kRadix - 1)] + i;
+        const long long dest = sh_goff[((k2 - row_base) >> S.shift) & (kRadix - 1)] + i;
         if (dest >= 0 && dest < S.n) {
             S.keys_out[dest] = k2;
             S.vals_out[dest] = sh_vals[i];
@@ -187,31 +197,80 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     }
 }
 
-// Exclusive scan of each pass's 256 digit counts (one block per pass).
-__global__ void digit_scan_kernel(const uint32_t* hist, uint32_t* base) {
-    __shared__ int64_t sh[33];
-    const int p = blockIdx.x, d = threadIdx.x;
-    int64_t total;
-    const int64_t ex = block_excl_scan(hist[p * kRadix + d], sh, &total);
-    base[p * kRadix + d] = static_cast<uint32_t>(ex);
+// Digit histograms of every pass, per table. Each block streams a contiguous
+// range of tiles, so its shared histogram changes table only a few times.
+__global__ void __launch_bounds__(256) sort_hist_kernel(const uint32_t* keys, const Chunk* tiles,
+                                                        const int64_t* num_tiles,
+                                                        const TableDev* tables, int passes,
+                                                        uint32_t* hist) {
+    __shared__ uint32_t sh[4 * kRadix];
+    const int64_t nt = *num_tiles;
+    const int64_t per = (nt + gridDim.x - 1) / gridDim.x;
+    const int64_t lo = static_cast<int64_t>(blockIdx.x) * per, hi = min64(lo + per, nt);
+    int cur = -1;
+    for (int i = threadIdx.x; i < 4 * kRadix; i += blockDim.x) sh[i] = 0;
+    __syncthreads();
+    for (int64_t j = lo; j < hi; ++j) {
+        const Chunk tc = tiles[j];
+        if (tc.table != cur) {  // uniform across the block
+            __syncthreads();    // every count of the previous table has landed
+            if (cur >= 0) {
+                for (int i = threadIdx.x; i < passes * kRadix; i += blockDim.x) {
+                    if (sh[i]) atomicAdd(hist + static_cast<int64_t>(cur) * passes * kRadix + i, sh[i]);
+                    sh[i] = 0;
+                }
+            }
+            __syncthreads();    // the flush is done before new counts start
+            cur = tc.table;
+        }
+        const uint32_t rb = static_cast<uint32_t>(tables[cur].row_base);
+        const int len = static_cast<int>(tc.len & 0x7fffffffu);
+        for (int i = threadIdx.x; i < len; i += blockDim.x) {
+            const uint32_t r = __ldg(keys + tc.k0 + i) - rb;
+            for (int p = 0; p < passes; ++p) atomicAdd(&sh[p * kRadix + ((r >> (8 * p)) & 255u)], 1u);
+        }
+    }
+    __syncthreads();
+    if (cur >= 0)
+        for (int i = threadIdx.x; i < passes * kRadix; i += blockDim.x)
+            if (sh[i]) atomicAdd(hist + static_cast<int64_t>(cur) * passes * kRadix + i, sh[i]);
 }
 
-int64_t sort_num_tiles(int64_t n) { return (n + kSortTile - 1) / kSortTile; }
+// First output position of each digit of each pass: the table's first position
+// plus the exclusive scan of that pass's digit counts (one block per table).
+__global__ void sort_base_kernel(const uint32_t* hist, const int64_t* table_pos, int passes,
+                                 uint32_t* base) {
+    __shared__ int64_t sh[33];
+    const int t = blockIdx.x, d = threadIdx.x;
+    for (int p = 0; p < passes; ++p) {
+        const int64_t i = (static_cast<int64_t>(t) * passes + p) * kRadix + d;
+        int64_t total;
+        const int64_t ex = block_excl_scan(hist[i], sh, &total);
+        base[i] = static_cast<uint32_t>(table_pos[t] + ex);
+    }
+}
 
-void launch_digit_scan(const uint32_t* hist, uint32_t* base, int passes, cudaStream_t s) {
-    digit_scan_kernel<<<passes, kRadix, 0, s>>>(hist, base);
+void launch_sort_hist(const uint32_t* keys, const Chunk* tiles, const int64_t* num_tiles,
+                      int64_t tile_bound, const TableDev* tables, int passes, uint32_t* hist,
+                      int num_sms, cudaStream_t s) {
+    const int grid = static_cast<int>(max64(1, min64(tile_bound, static_cast<int64_t>(num_sms) * 4)));
+    sort_hist_kernel<<<grid, 256, 0, s>>>(keys, tiles, num_tiles, tables, passes, hist);
+}
+
+void launch_sort_bases(const uint32_t* hist, const int64_t* table_pos, int T, int passes,
+                       uint32_t* base, cudaStream_t s) {
+    sort_base_kernel<<<T, kRadix, 0, s>>>(hist, table_pos, passes, base);
 }
 
 constexpr int kSortDynSmem = 3 * kSortTile * sizeof(uint32_t);  // 48 KB
 
-void launch_onesweep(const SortPass& S, cudaStream_t s) {
+void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     static bool configured = false;
     if (!configured) {
         cudaFuncSetAttribute(onesweep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSortDynSmem);
         configured = true;
     }
-    const int64_t tiles = sort_num_tiles(S.n);
-    onesweep_kernel<<<static_cast<unsigned>(tiles), kSortThreads, kSortDynSmem, s>>>(S);
+    onesweep_kernel<<<static_cast<unsigned>(max64(tile_bound, 1)), kSortThreads, kSortDynSmem, s>>>(S);
 }
 
 }  // namespace cbtbe

@@ -87,9 +87,10 @@ def sort_bytes(n: int, passes: int) -> int:
 
 
 def radix_passes(rows) -> int:
-    total = int(sum(rows))
+    """8-bit passes over the row number of the largest table (ranges sorted per table)."""
+    largest = max(1, int(max(rows)))
     bits = 1
-    while bits < 32 and (1 << bits) < total:
+    while bits < 32 and (1 << bits) < largest:
         bits += 1
     return (bits + 7) // 8
 

@@ -27,11 +27,12 @@ def test_forward_and_backward_bytes_by_hand():
     assert metrics.forward_unique_bytes(c, [3, 1]) == f["total"] - f["rows"] + 3 * 8 + 1 * 16
 
 
-def test_radix_passes_follow_key_bits():
+def test_radix_passes_follow_row_bits():
     assert metrics.radix_passes([256]) == 1
     assert metrics.radix_passes([257]) == 2
-    assert metrics.radix_passes([5_000_000] * 100) == 4   # 29-bit keys
-    assert metrics.radix_passes([100_000] * 8) == 3       # 20-bit keys
+    assert metrics.radix_passes([5_000_000] * 100) == 3   # 23-bit rows, per-table ranges
+    assert metrics.radix_passes([100_000] * 8) == 3       # 17-bit rows
+    assert metrics.radix_passes([1000, 70000]) == 3       # the largest table decides
     assert metrics.sort_bytes(10, 3) == 480
 
 
