@@ -225,9 +225,18 @@ __global__ void __launch_bounds__(256) sort_hist_kernel(const uint32_t* keys, co
         }
         const uint32_t rb = static_cast<uint32_t>(tables[cur].row_base);
         const int len = static_cast<int>(tc.len & 0x7fffffffu);
-        for (int i = threadIdx.x; i < len; i += blockDim.x) {
-            const uint32_t r = __ldg(keys + tc.k0 + i) - rb;
-            for (int p = 0; p < passes; ++p) atomicAdd(&sh[p * kRadix + ((r >> (8 * p)) & 255u)], 1u);
+        // All of the tile's loads first, then the counts.
+        uint32_t r[kSortItems];
+#pragma unroll
+        for (int k = 0; k < kSortItems; ++k) {
+            const int i = threadIdx.x + k * 256;
+            r[k] = i < len ? __ldg(keys + tc.k0 + i) - rb : 0u;
+        }
+#pragma unroll
+        for (int k = 0; k < kSortItems; ++k) {
+            if (threadIdx.x + k * 256 >= len) break;
+            for (int p = 0; p < passes; ++p)
+                atomicAdd(&sh[p * kRadix + ((r[k] >> (8 * p)) & 255u)], 1u);
         }
     }
     __syncthreads();
