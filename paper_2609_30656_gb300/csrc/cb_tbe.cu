@@ -226,6 +226,9 @@ Problem make_problem(const cb_tbe* h, int32_t B, const void* indices, int64_t n,
 Plan make_plan(const cb_tbe* h, const Workspace& w, bool bwd, int64_t chunk_len) {
     Plan Q;
     Q.chunk_len = static_cast<int32_t>(chunk_len);
+    // Chunk boundaries move to the end of the bag / run they cut unless it is
+    // longer than this, so only heavy bags and hot rows are split.
+    Q.snap_cap = static_cast<int32_t>(bwd ? chunk_len : 4 * chunk_len);
     Q.num_classes = static_cast<int32_t>(bwd ? h->bwd_classes.size() : h->fwd_classes.size());
     Q.class_tables = bwd ? h->d_bwd_class_tables : h->d_fwd_class_tables;
     Q.class_table_start = bwd ? h->d_bwd_class_start : h->d_fwd_class_start;
@@ -533,6 +536,7 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
     // (2) radix sort of each table's range, 8 bits of the row number per pass
     Plan SQ;
     SQ.chunk_len = static_cast<int32_t>(kSortTileKeys);
+    SQ.snap_cap = 0;
     SQ.num_classes = 1;
     SQ.class_tables = h->d_all_tables;
     SQ.class_table_start = h->d_all_start;

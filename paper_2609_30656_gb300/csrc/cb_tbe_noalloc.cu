@@ -197,6 +197,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
     } else {
         Plan Q;
         Q.chunk_len = static_cast<int32_t>(kChunk);
+        Q.snap_cap = static_cast<int32_t>(4 * kChunk);  // as the handle's forward
         Q.num_classes = static_cast<int32_t>(nc);
         Q.class_tables = reinterpret_cast<const int32_t*>(base + o_ct);
         Q.class_table_start = reinterpret_cast<const int32_t*>(base + o_cs);

@@ -316,26 +316,32 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
 
 // ---------------------------------------------------------------- (6) fix-up
 
+// Runs split over chunks (hot rows longer than the snap cap): each warp scans
+// 32 chunks at a time for tail pieces and combines each such run in fp64.
 __global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(const __grid_constant__ Problem P,
                                                                  const __grid_constant__ Plan Q,
                                                                  const __grid_constant__ BwdOut O) {
     if (*O.cap_fail) return;
     const int lane = threadIdx.x & 31;
     const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
-    const int64_t j = warp_id_global();
-    if (j >= total) return;
-    const int64_t seg = Q.tail_owner[j];
-    if (seg < 0) return;
-    const int t = Q.chunks[j].table;
-    const TableDev& td = P.tables[t];
-    const int64_t e = O.seg_start[seg + 1];
-    const int64_t m = pieces_after(Q, j, e, total);
-    float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
-    combine_pieces(Q, j, m, td.dim, P.dmax, lane, [&](int x0, double (&acc)[4]) {
-        *reinterpret_cast<float4*>(dst + x0) =
-            make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
-                        static_cast<float>(acc[2]), static_cast<float>(acc[3]));
-    });
+    for (int64_t base = warp_id_global() * 32; base < total; base += warps_in_grid() * 32) {
+        const int64_t mine = base + lane < total ? Q.tail_owner[base + lane] : -1;
+        for (uint32_t mask = __ballot_sync(kFull, mine >= 0); mask; mask &= mask - 1) {
+            const int b = __ffs(mask) - 1;
+            const int64_t j = base + b;
+            const int64_t seg = __shfl_sync(kFull, mine, b);
+            const int t = Q.chunks[j].table;
+            const TableDev& td = P.tables[t];
+            const int64_t e = O.seg_start[seg + 1];
+            const int64_t m = pieces_after(Q, j, e, total);
+            float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
+            combine_pieces(Q, j, m, td.dim, P.dmax, lane, [&](int x0, double (&acc)[4]) {
+                *reinterpret_cast<float4*>(dst + x0) =
+                    make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                                static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+            });
+        }
+    }
 }
 
 // ---------------------------------------------------------------- launchers
@@ -404,9 +410,9 @@ void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const f
 
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s) {
-    (void)num_sms;  // one warp per chunk
-    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
-    bwd_fixup_kernel<<<static_cast<unsigned>(max64(need, 1)), kWarpThreads, 0, s>>>(P, Q, O);
+    const int64_t need = (chunk_bound + kWarpThreads - 1) / kWarpThreads;  // 32 chunks per warp
+    const int grid = static_cast<int>(max64(1, min64(need, static_cast<int64_t>(num_sms) * 8)));
+    bwd_fixup_kernel<<<grid, kWarpThreads, 0, s>>>(P, Q, O);
 }
 
 }  // namespace cbtbe

@@ -84,6 +84,7 @@ struct Problem {
 
 struct Plan {
     int32_t chunk_len;
+    int32_t snap_cap;                  // segments up to this long are never split (0: no snapping)
     int32_t num_classes;
     const int32_t* class_tables;       // [T] table ids grouped by kernel class
     const int32_t* class_table_start;  // [num_classes + 1]

@@ -63,12 +63,60 @@ __global__ void __launch_bounds__(1024) plan_tables_kernel(Problem P, Plan Q) {
     }
 }
 
+// Segment bounds around a position: the first bag of table t starting at or
+// after x (lower bound over the table's offsets), or the run of sorted ids
+// containing x.
+__device__ __forceinline__ int64_t bag_lower_bound(const Problem& P, int t, int64_t x) {
+    const int64_t blo = static_cast<int64_t>(t) * P.B, bhi = blo + P.B;
+    int64_t a = blo, b = bhi + 1;
+    while (a < b) {
+        const int64_t m = (a + b) >> 1;
+        if (load_index(P.offsets, m, P.is32) < x) a = m + 1; else b = m;
+    }
+    return a;  // in [blo, bhi + 1]
+}
+
+__device__ __forceinline__ int64_t run_containing(const uint32_t* seg_start, int64_t U, int64_t x) {
+    int64_t a = 0, b = U + 1;
+    while (a < b) {
+        const int64_t m = (a + b) >> 1;
+        if (static_cast<int64_t>(seg_start[m]) <= x) a = m + 1; else b = m;
+    }
+    return max64(a - 1, 0);
+}
+
+// A chunk boundary at x moves to the end of the segment it falls in, unless
+// that segment is longer than the cap: short bags and runs are then never
+// split, and only heavy ones leave pieces for the fix-up. Monotone in x, so
+// consecutive chunks stay contiguous (a chunk may come out empty).
+__device__ __forceinline__ int64_t snap(const Problem& P, const Plan& Q, int mode, int t,
+                                        const uint32_t* seg_start, int64_t U, int64_t x,
+                                        int64_t p0, int64_t p1) {
+    if (Q.snap_cap <= 0 || x <= p0 || x >= p1) return x;
+    if (mode == 0) {
+        const int64_t a = bag_lower_bound(P, t, x);
+        const int64_t bhi = static_cast<int64_t>(t) * P.B + P.B;
+        if (a > bhi) return x;
+        const int64_t e = load_index(P.offsets, a, P.is32);
+        if (e == x || a == static_cast<int64_t>(t) * P.B) return x;
+        const int64_t s0 = load_index(P.offsets, a - 1, P.is32);
+        return (e - s0 <= Q.snap_cap && e <= p1) ? e : x;
+    }
+    if (mode == 1) {
+        const int64_t u = run_containing(seg_start, U, x);
+        const int64_t s0 = seg_start[u], e = seg_start[u + 1];
+        if (s0 == x) return x;
+        return (e - s0 <= Q.snap_cap && e <= p1) ? e : x;
+    }
+    return x;
+}
+
 // mode 0: first = the bag touching the chunk start (forward, key generation).
 // mode 1: first = the run of sorted ids containing the chunk start (reduce).
-// mode 2: tiles only (radix sort), first left at 0.
+// mode 2: tiles only (radix sort), first left at 0, no snapping.
 __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* seg_start,
                                    const int64_t* num_unique) {
-    const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     const int64_t C = Q.chunk_len;
     const int64_t U = mode == 1 ? *num_unique : 0;
@@ -83,34 +131,24 @@ __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* 
         const int t = Q.class_tables[lo];
         const int64_t local = j - Q.ord_chunk_base[lo];
         const int64_t p0 = Q.table_pos[t];
-        const int64_t p1 = max(p0, Q.table_pos[t + 1]);
-        const int64_t nch = max(static_cast<int64_t>(1), (p1 - p0 + C - 1) / C);
-        const int64_t k0 = min(p0 + local * C, p1);
-        const int64_t len = min(C, p1 - k0);
+        const int64_t p1 = max64(p0, Q.table_pos[t + 1]);
+        const int64_t nch = max64(1, (p1 - p0 + C - 1) / C);
         const bool last = local >= nch - 1;
+        const int64_t x0 = min64(p0 + local * C, p1);
+        const int64_t x1 = last ? p1 : min64(p0 + (local + 1) * C, p1);
+        const int64_t k0 = mode == 2 ? x0 : snap(P, Q, mode, t, seg_start, U, x0, p0, p1);
+        const int64_t k1 = mode == 2 || last ? x1 : snap(P, Q, mode, t, seg_start, U, x1, p0, p1);
+        const int64_t len = max64(0, k1 - k0);
         int64_t first = 0;
-        if (mode == 2) {
-            // tiles only (radix sort): no first segment needed
-        } else if (mode == 0) {
-            // First bag b of table t with offsets[b] >= k0 (lower bound over the
-            // table's B + 1 offsets); the chunk starts in the bag before it unless
-            // a bag starts exactly at k0.
+        if (mode == 0) {
+            // First bag of table t touching k0: the bag starting exactly at k0
+            // if any (the first of equal starts), else the one containing k0.
             const int64_t blo = static_cast<int64_t>(t) * P.B, bhi = blo + P.B;
-            int64_t a = blo, b = bhi + 1;
-            while (a < b) {
-                const int64_t m = (a + b) >> 1;
-                if (load_index(P.offsets, m, P.is32) < k0) a = m + 1; else b = m;
-            }
+            const int64_t a = bag_lower_bound(P, t, k0);
             first = (a <= bhi && load_index(P.offsets, a, P.is32) == k0) ? a : a - 1;
-            first = min(max(first, blo), bhi);
-        } else {
-            // Last run u with seg_start[u] <= k0.
-            int64_t a = 0, b = U + 1;
-            while (a < b) {
-                const int64_t m = (a + b) >> 1;
-                if (static_cast<int64_t>(seg_start[m]) <= k0) a = m + 1; else b = m;
-            }
-            first = max(a - 1, static_cast<int64_t>(0));
+            first = min64(max64(first, blo), bhi);
+        } else if (mode == 1) {
+            first = run_containing(seg_start, U, k0);
         }
         Chunk ch;
         ch.k0 = k0;
