@@ -81,6 +81,9 @@ struct Workspace {
     int64_t* float_base = nullptr;
     int64_t* num_unique = nullptr;
     int* cap_fail = nullptr;
+    int4* heavy = nullptr;
+    uint32_t* heavy_count = nullptr;
+    int64_t max_heavy = 0;
     int64_t sort_tiles = 0;
     size_t status_bytes = 0;
 };
@@ -177,6 +180,9 @@ size_t layout(const cb_tbe* h, int64_t B, int64_t n, char* base, Workspace* w) {
     ws.float_base = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
     ws.num_unique = static_cast<int64_t*>(take(sizeof(int64_t)));
     ws.cap_fail = static_cast<int*>(take(sizeof(int)));
+    ws.max_heavy = max_chunks / 32 + 1;  // a heavy run owns more than 32 chunks
+    ws.heavy = static_cast<int4*>(take(sizeof(int4) * ws.max_heavy));
+    ws.heavy_count = static_cast<uint32_t*>(take(sizeof(uint32_t)));
     if (w) *w = ws;
     return off;
 }
@@ -591,6 +597,9 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
     O.table_first = w.table_first;
     O.float_base = w.float_base;
     O.cap_fail = w.cap_fail;
+    O.heavy = w.heavy;
+    O.heavy_count = w.heavy_count;
+    O.max_heavy = w.max_heavy;
     O.unique_ids = g->unique_ids;
     O.table_offsets = g->table_offsets;
     O.grad_offsets = g->grad_offsets;
@@ -613,7 +622,7 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
             h->launches += 1;
         }
         launch_bwd_fixup(P, Q, O, bound, h->num_sms, stream);
-        h->launches += 1;
+        h->launches += 2;
     }
     record(h, h->ev_bwd[4], stream);
     h->bwd_timed = (h->flags & CB_TIMING) != 0;

@@ -317,7 +317,17 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
 // ---------------------------------------------------------------- (6) fix-up
 
 // Runs split over chunks (hot rows longer than the snap cap): each warp scans
-// 32 chunks at a time for tail pieces and combines each such run in fp64.
+// 32 chunks at a time for tail pieces and combines each such run in fp64. Runs
+// spread over more than kHeavyPieces chunks go to a list that bwd_heavy_kernel
+// combines with a whole block each.
+constexpr int64_t kHeavyPieces = 32;
+
+__device__ __forceinline__ void store_grad4(float* dst, int x0, const double (&acc)[4]) {
+    *reinterpret_cast<float4*>(dst + x0) =
+        make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                    static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+}
+
 __global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(const __grid_constant__ Problem P,
                                                                  const __grid_constant__ Plan Q,
                                                                  const __grid_constant__ BwdOut O) {
@@ -330,17 +340,68 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(const __grid_co
             const int b = __ffs(mask) - 1;
             const int64_t j = base + b;
             const int64_t seg = __shfl_sync(kFull, mine, b);
-            const int t = Q.chunks[j].table;
-            const TableDev& td = P.tables[t];
             const int64_t e = O.seg_start[seg + 1];
             const int64_t m = pieces_after(Q, j, e, total);
+            if (m > kHeavyPieces) {
+                if (lane == 0) {
+                    const uint32_t slot = atomicAdd(O.heavy_count, 1u);
+                    if (slot < O.max_heavy)
+                        O.heavy[slot] = make_int4(static_cast<int>(j), static_cast<int>(seg),
+                                                  static_cast<int>(m), 0);
+                }
+                continue;
+            }
+            const int t = Q.chunks[j].table;
+            const TableDev& td = P.tables[t];
             float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
-            combine_pieces(Q, j, m, td.dim, P.dmax, lane, [&](int x0, double (&acc)[4]) {
-                *reinterpret_cast<float4*>(dst + x0) =
-                    make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
-                                static_cast<float>(acc[2]), static_cast<float>(acc[3]));
-            });
+            combine_pieces(Q, j, m, td.dim, P.dmax, lane,
+                           [&](int x0, double (&acc)[4]) { store_grad4(dst, x0, acc); });
         }
+    }
+}
+
+// One heavy run per block: warp w adds pieces w, w + 8, ... (lanes own columns),
+// then the warps' partial sums meet in shared memory in warp order, after the
+// tail piece. The order is fixed, so the result is deterministic.
+__global__ void __launch_bounds__(kWarpThreads) bwd_heavy_kernel(const __grid_constant__ Problem P,
+                                                                 const __grid_constant__ Plan Q,
+                                                                 const __grid_constant__ BwdOut O) {
+    __shared__ double sh[kWarpThreads / 32][512];
+    if (*O.cap_fail) return;
+    const uint32_t count = min64(*O.heavy_count, O.max_heavy);
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    constexpr int kWarps = kWarpThreads / 32;
+    for (uint32_t h = blockIdx.x; h < count; h += gridDim.x) {
+        const int4 rec = O.heavy[h];
+        const int64_t j = rec.x, seg = rec.y, m = rec.z;
+        const int t = Q.chunks[j].table;
+        const TableDev& td = P.tables[t];
+        const float* head = Q.carry_head + (j + 1) * P.dmax;
+        for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
+            double acc[4] = {0.0, 0.0, 0.0, 0.0};
+#pragma unroll 8
+            for (int64_t i = w; i < m; i += kWarps) {
+                const float4 v = *reinterpret_cast<const float4*>(head + i * P.dmax + x0);
+                acc[0] += v.x;
+                acc[1] += v.y;
+                acc[2] += v.z;
+                acc[3] += v.w;
+            }
+            for (int x = 0; x < 4; ++x) sh[w][x0 + x] = acc[x];
+        }
+        __syncthreads();
+        if (w == 0) {
+            float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
+            const float* tail = Q.carry_tail + j * P.dmax;
+            for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
+                const float4 a = *reinterpret_cast<const float4*>(tail + x0);
+                double acc[4] = {a.x, a.y, a.z, a.w};
+                for (int ww = 0; ww < kWarps; ++ww)
+                    for (int x = 0; x < 4; ++x) acc[x] += sh[ww][x0 + x];
+                store_grad4(dst, x0, acc);
+            }
+        }
+        __syncthreads();
     }
 }
 
@@ -410,9 +471,12 @@ void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const f
 
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s) {
+    cudaMemsetAsync(O.heavy_count, 0, sizeof(uint32_t), s);
     const int64_t need = (chunk_bound + kWarpThreads - 1) / kWarpThreads;  // 32 chunks per warp
     const int grid = static_cast<int>(max64(1, min64(need, static_cast<int64_t>(num_sms) * 8)));
     bwd_fixup_kernel<<<grid, kWarpThreads, 0, s>>>(P, Q, O);
+    const int hgrid = static_cast<int>(max64(1, min64(O.max_heavy, static_cast<int64_t>(num_sms) * 4)));
+    bwd_heavy_kernel<<<hgrid, kWarpThreads, 0, s>>>(P, Q, O);
 }
 
 }  // namespace cbtbe

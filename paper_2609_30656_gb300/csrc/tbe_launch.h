@@ -48,6 +48,9 @@ struct BwdOut {
     int64_t* table_first;        // [T + 1]
     int64_t* float_base;         // [T + 1]
     int* cap_fail;
+    int4* heavy;                 // [max_heavy] runs left for the block-wide combine
+    uint32_t* heavy_count;       // zeroed before the fix-up
+    int64_t max_heavy;
     // caller's buffers
     int64_t* unique_ids;
     int64_t* table_offsets;
