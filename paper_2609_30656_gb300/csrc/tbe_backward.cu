@@ -220,6 +220,8 @@ struct BwdPolicy {
     static constexpr int kVpl = VPL;
     static constexpr int kUnroll = CB_REDUCE_ROWS / VPL > 0 ? CB_REDUCE_ROWS / VPL : 1;
     static constexpr bool kWeighted = PACKED;
+    static constexpr bool kUnrollGroups = CB_REDUCE_UNROLL_GROUPS;
+    static constexpr bool kFastBatch = CB_REDUCE_FAST_BATCH;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;
@@ -258,15 +260,22 @@ struct BwdPolicy {
         const int64_t b = bag - bag_lo;
         a = (b >= 0 && b < P.B) ? static_cast<uint32_t>(b) : kInvalid;
     }
-    __device__ __forceinline__ void emit(int32_t seg, int32_t, bool started, bool ends,
+    static constexpr bool kEmptySegments = false;
+    // Row id and float offset of a run that begins in this chunk.
+    __device__ __forceinline__ void seg_meta(int32_t seg) const {
+        O.unique_ids[seg] = __ldg(O.uniq + seg);
+        O.grad_offsets[seg] = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
+    }
+    __device__ __forceinline__ void put_empty(int32_t, int, bool) const {}
+    __device__ __forceinline__ void emit(int32_t seg, int32_t L, bool started, bool ends,
                                          float (&tot)[VPL][4], int v, bool group0) const {
-        const int lane = threadIdx.x & 31;
+        if (started && (threadIdx.x & 31) == 0) seg_meta(seg);
+        put(seg, L, started, ends, tot, v, group0);
+    }
+    __device__ __forceinline__ void put(int32_t seg, int32_t, bool started, bool ends,
+                                        float (&tot)[VPL][4], int v, bool group0) const {
         const int64_t fo = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
-        if (started && lane == 0) {
-            O.unique_ids[seg] = __ldg(O.uniq + seg);
-            O.grad_offsets[seg] = fo;
-            if (!ends) Q.tail_owner[chunk] = seg;
-        }
+        if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = seg;
         if (!group0) return;
         float* dst;
         if (started && ends) dst = O.grads + fo;
@@ -310,7 +319,12 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
         c.row_vecs = td.grad_vecs;
         c.last = false;
         if (lane == 0) Q.tail_owner[j] = -1;
-        walk_chunk<BwdPolicy<VPL, PACKED>, GC>(pol, c, P.zero_row, lane);
+        if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
+            __shared__ EndSlot slots[kWarpThreads / 32][32];
+            walk_rows<BwdPolicy<VPL, PACKED>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+        } else {
+            walk_chunk<BwdPolicy<VPL, PACKED>, GC>(pol, c, P.zero_row, lane);
+        }
     }
 }
 

@@ -23,6 +23,8 @@ struct FwdPolicy {
     static constexpr int kVpl = VPL;
     static constexpr int kUnroll = CB_WALK_ROWS / VPL > 0 ? CB_WALK_ROWS / VPL : 1;
     static constexpr bool kWeighted = WEIGHTED;
+    static constexpr bool kUnrollGroups = CB_WALK_UNROLL_GROUPS;
+    static constexpr bool kFastBatch = CB_WALK_FAST_BATCH;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;
@@ -54,6 +56,20 @@ struct FwdPolicy {
         } else {
             a = static_cast<uint32_t>(x.r);
         }
+    }
+    static constexpr bool kEmptySegments = true;
+    __device__ __forceinline__ void seg_meta(int32_t) const {}
+    __device__ __forceinline__ void put(int32_t bag, int32_t L, bool started, bool ends,
+                                        float (&tot)[VPL][kElems], int v, bool group0) const {
+        emit(bag, L, started, ends, tot, v, group0);
+    }
+    // An empty bag pools to zeros (one vector per lane).
+    __device__ __forceinline__ void put_empty(int32_t bag, int v, bool group0) const {
+        if (!group0) return;
+        float4* d4 = reinterpret_cast<float4*>(out + static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff +
+                                               v * kElems);
+#pragma unroll
+        for (int x = 0; x < kElems / 4; ++x) d4[x] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
     __device__ __forceinline__ void emit(int32_t bag, int32_t L, bool started, bool ends,
                                          float (&tot)[VPL][kElems], int v, bool group0) const {
@@ -113,7 +129,12 @@ __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
         c.row_vecs = td.row_vecs;
         c.last = (ch.len >> 31) != 0;
         if (lane == 0) Q.tail_owner[j] = -1;
-        walk_chunk<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane);
+        if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
+            __shared__ EndSlot slots[kWarpThreads / 32][32];
+            walk_rows<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+        } else {
+            walk_chunk<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane);
+        }
     }
 }
 

@@ -18,6 +18,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
+#include <type_traits>
 
 #include "cb_tbe.h"
 
@@ -36,6 +37,26 @@ constexpr int kWarpThreads = 256;  // block size of the warp-per-chunk kernels
 #endif
 #ifndef CB_REDUCE_ROWS
 #define CB_REDUCE_ROWS 8
+#endif
+// Row-walker code shape, per kernel (measured on cfg5): the forward keeps one
+// copy of the segment-end code per batch (unrolling it over the load groups
+// overflowed the instruction cache and doubled the gather time) and unrolls
+// only batches with no segment end; the backward reduce, whose segment-end
+// code is small, unrolls every batch.
+#ifndef CB_WALK_UNROLL_GROUPS
+#define CB_WALK_UNROLL_GROUPS 0
+#endif
+#ifndef CB_WALK_FAST_BATCH
+#define CB_WALK_FAST_BATCH 1
+#endif
+#ifndef CB_REDUCE_UNROLL_GROUPS
+#define CB_REDUCE_UNROLL_GROUPS 1
+#endif
+#ifndef CB_REDUCE_FAST_BATCH
+#define CB_REDUCE_FAST_BATCH 0
+#endif
+#ifndef CB_ROW_WALKER
+#define CB_ROW_WALKER 1  // 0: every layout takes the general walker (walk_chunk)
 #endif
 constexpr int64_t kNoSeg = INT64_MAX;
 
@@ -403,6 +424,227 @@ __device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const ui
         flush();
         if (!done) break;
         advance();
+    }
+}
+
+// ---------------------------------------------------------------- the row walker
+//
+// walk_rows has walk_chunk's contract for the common layout, one 16-byte vector
+// per lane and G = 32 / V rows per warp step fixed at compile time, and is built
+// around batches of 32 item positions. Before a batch's rows are loaded, the
+// warp finds every segment ending inside the batch from a window of 32 segment
+// ends (one per lane): the positions of those ends become a 32-bit mask, and
+// their segment numbers go to a per-warp list in shared memory, in order. Adding
+// a row then costs a shuffle, one multiply-add for its address, the load and
+// the adds, and the mask is tested once per group of loads; a segment end costs
+// one list read and the store of the sum. Empty segments (empty bags) are
+// written out during the scan. Pol additionally supplies:
+//   static constexpr bool kEmptySegments    segments may be empty
+//   static constexpr bool kUnrollGroups     unroll a batch's load groups
+//   static constexpr bool kFastBatch        separate unrolled path for batches
+//                                            with no segment end
+//   void put(seg, len, started, ends, tot, v, is_group0)   emit without the
+//                                            per-segment metadata
+//   void seg_meta(seg)                       metadata of a segment that began in
+//                                            this chunk (once per segment; lanes
+//                                            may call it for different segments
+//                                            at the same time)
+//   void put_empty(seg, v, is_group0)        the output of an empty segment
+
+struct EndSlot {
+    int32_t seg;
+    int32_t len;  // segment length, or -1 when it began in an earlier chunk
+};
+
+template <class Pol, int G>
+__device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uint4* zero_row,
+                                          int lane, EndSlot* slots) {
+    static_assert(G == 1 || G == 2 || G == 4 || G == 8, "rows per warp step");
+    static_assert(Pol::kVpl == 1, "one vector per lane");
+    constexpr int E = Pol::kElems;
+    constexpr int V = 32 / G;
+    constexpr int kSteps = 32 / G;                                      // row steps per batch
+    constexpr int UG = Pol::kUnroll < kSteps ? Pol::kUnroll : kSteps;  // row steps per load group
+    constexpr int kGroupItems = UG * G;
+    constexpr uint32_t kGroupMask = kGroupItems == 32 ? kFull : (1u << kGroupItems) - 1u;
+    constexpr uint32_t kStepMask = (1u << G) - 1u;
+    constexpr bool W = Pol::kWeighted;
+    constexpr bool kTwoLevel = Pol::kDtype == CB_F32;
+    constexpr int kGroupUnroll = Pol::kUnrollGroups ? 32 / kGroupItems : 1;
+    const int g = lane / V;
+    const int v = lane - g * V;
+    const int32_t len = c.len;
+    const char* lane_base = reinterpret_cast<const char*>(pol.base + v);
+    const uint32_t row_bytes = pol.stride * 16u;
+    const uint4* zrow = zero_row + v;
+    const uint32_t below = (1u << lane) - 1u;
+
+    float ain[E], aout[kTwoLevel ? E : 1];
+#pragma unroll
+    for (int x = 0; x < E; ++x) ain[x] = 0.f;
+#pragma unroll
+    for (int x = 0; x < (kTwoLevel ? E : 1); ++x) aout[x] = 0.f;
+
+    // Window: lane j holds the relative end of segment seg + j.
+    int32_t seg = c.first;
+    int32_t s_cur = seg < c.seg_hi ? rel_pos(pol.seg_begin(seg), c.k0) : kRelHi;
+    int32_t my_end = seg + lane < c.seg_hi ? rel_pos(pol.seg_end(seg + lane), c.k0) : kRelHi;
+    uint32_t mask = 0;
+
+    // Segments ending at or before `bend` (the batch starts at `base`) leave the
+    // window: non-empty ones are listed and marked in `mask`, empty ones owned
+    // by this chunk are written out. Ends are non-decreasing, so the finished
+    // segments are a prefix of the window.
+    auto scan = [&](int32_t base, int32_t bend) {
+        __syncwarp();  // every lane is done reading the previous batch's list
+        mask = 0;
+        int nend = 0;
+        for (;;) {
+            int32_t my_beg = __shfl_up_sync(kFull, my_end, 1);
+            if (lane == 0) my_beg = s_cur;
+            const bool nonempty = my_end > my_beg;
+            const bool done = my_end <= bend && (nonempty || my_end < len || c.last);
+            const uint32_t dm = __ballot_sync(kFull, done);
+            const uint32_t ne = __ballot_sync(kFull, done && nonempty);
+            if (done && nonempty) {
+                // (index masked: malformed offsets, which are reported, can
+                // break the prefix property but never reach past the list)
+                slots[(nend + __popc(ne & below)) & 31] = EndSlot{seg + lane, my_beg >= 0 ? my_end - my_beg : -1};
+                if (my_beg >= 0) pol.seg_meta(seg + lane);
+            }
+            if constexpr (Pol::kEmptySegments) {
+                for (uint32_t em = dm & ~ne; em; em &= em - 1) pol.put_empty(seg + __ffs(em) - 1, v, g == 0);
+            }
+            mask |= __reduce_or_sync(kFull, (done && nonempty) ? 1u << ((my_end - base - 1) & 31) : 0u);
+            nend += __popc(ne);
+            const int nd = __popc(dm);
+            if (nd == 0) break;
+            const int32_t last_end = __shfl_sync(kFull, my_end, nd - 1);
+            const int32_t moved = __shfl_down_sync(kFull, my_end, nd & 31);
+            s_cur = last_end;
+            seg += nd;
+            my_end = lane + nd < 32 ? moved
+                                    : (seg + lane < c.seg_hi ? rel_pos(pol.seg_end(seg + lane), c.k0) : kRelHi);
+            // A full window that finished before `bend` leaves more to find; at
+            // the chunk end, so may one that finished exactly there (empty
+            // segments at the end of the table's last chunk).
+            if (nd < 32 || (last_end >= bend && !(Pol::kEmptySegments && bend == len))) break;
+        }
+        __syncwarp();
+    };
+
+    auto flush = [&](const EndSlot s, bool ends) {
+        // Kept inside this chunk's segment range whatever the list holds.
+        const int32_t sseg = min(max(s.seg, c.first), c.seg_hi - 1);
+        float tot[1][E];
+#pragma unroll
+        for (int x = 0; x < E; ++x) tot[0][x] = kTwoLevel ? aout[x] + ain[x] : ain[x];
+#pragma unroll
+        for (int off = V; off < 32; off <<= 1)
+#pragma unroll
+            for (int x = 0; x < E; ++x) tot[0][x] += __shfl_xor_sync(kFull, tot[0][x], off);
+        pol.put(sseg, s.len, s.len >= 0, ends, tot, v, g == 0);
+#pragma unroll
+        for (int x = 0; x < E; ++x) ain[x] = 0.f;
+#pragma unroll
+        for (int x = 0; x < (kTwoLevel ? E : 1); ++x) aout[x] = 0.f;
+    };
+
+    // One batch's rows: CLEAN = 32 valid items (no padding, no skipped item).
+    auto rows = [&](auto clean_tag, uint32_t my_a, float my_w, int nb) {
+        constexpr bool CLEAN = decltype(clean_tag)::value;
+        int ce = 0;
+#pragma unroll(kGroupUnroll)
+        for (int i0 = 0; i0 < 32; i0 += kGroupItems) {
+            if (!CLEAN && i0 >= nb) break;
+            uint4 buf[UG];
+            float wt[UG];
+#pragma unroll
+            for (int u = 0; u < UG; ++u) {
+                const int src = i0 + u * G + g;
+                const uint32_t a = __shfl_sync(kFull, my_a, src);
+                wt[u] = W ? __shfl_sync(kFull, my_w, src) : 1.f;
+                const uint4* p = reinterpret_cast<const uint4*>(lane_base + static_cast<uint64_t>(a) * row_bytes);
+                buf[u] = __ldg(CLEAN || a != kInvalid ? p : zrow);
+            }
+            const uint32_t m = (mask >> i0) & kGroupMask;
+            if (m == 0) {
+#pragma unroll
+                for (int u = 0; u < UG; ++u) accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                continue;
+            }
+#pragma unroll
+            for (int u = 0; u < UG; ++u) {
+                uint32_t mu = (m >> (u * G)) & kStepMask;
+                if (mu == 0) {
+                    accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                    continue;
+                }
+                // Segments end after item i0 + u*G + p for each set bit p; this
+                // group's item (p index g) belongs to the first of them with g <= p.
+                bool added = false;
+                do {
+                    const int p = __ffs(mu) - 1;
+                    if (!added && g <= p) {
+                        accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                        added = true;
+                    }
+                    flush(slots[ce++], true);
+                    mu &= mu - 1;
+                } while (mu);
+                if (!added) accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+            }
+        }
+    };
+
+    typename Pol::Raw nxt = Pol::none();
+    if (lane < len) nxt = pol.fetch(c.k0 + lane);
+    for (int32_t base = 0; base < len; base += 32) {
+        const int nb = min(32, len - base);
+        const typename Pol::Raw cur = nxt;
+        nxt = Pol::none();
+        if (base + 32 + lane < len) nxt = pol.fetch(c.k0 + base + 32 + lane);
+        uint32_t my_a = kInvalid;
+        float my_w = 0.f;
+        if (lane < nb) pol.decode(cur, my_a, my_w);
+        scan(base, base + nb);
+        const bool clean = __all_sync(kFull, my_a != kInvalid);
+        if (Pol::kFastBatch && clean && mask == 0) {
+            // The whole batch adds into the open segment: every load group
+            // unrolled, so loads of later groups overlap the adds of earlier ones.
+#pragma unroll
+            for (int i0 = 0; i0 < 32; i0 += kGroupItems) {
+#pragma unroll
+                for (int u = 0; u < UG; ++u) {
+                    const int src = i0 + u * G + g;
+                    const uint32_t a = __shfl_sync(kFull, my_a, src);
+                    const float w = W ? __shfl_sync(kFull, my_w, src) : 1.f;
+                    const uint4 x = __ldg(reinterpret_cast<const uint4*>(
+                        lane_base + static_cast<uint64_t>(a) * row_bytes));
+                    accumulate<Pol::kDtype, W>(ain, x, w);
+                }
+            }
+        } else if (clean) {
+            rows(std::true_type{}, my_a, my_w, nb);
+        } else {
+            rows(std::false_type{}, my_a, my_w, nb);
+        }
+        // Two-level summation: at most 32 / G terms per lane enter `ain` before
+        // it is folded into `aout`, which bounds the fp32 rounding error.
+        if (kTwoLevel) {
+#pragma unroll
+            for (int x = 0; x < E; ++x) {
+                aout[x] += ain[x];
+                ain[x] = 0.f;
+            }
+        }
+    }
+    // Empty segments at the chunk end (last chunk of a table), and chunks with
+    // no items; then the piece of the segment that runs past the chunk end.
+    scan(len, len);
+    if (seg < c.seg_hi && s_cur < len) {
+        if (s_cur >= 0 && lane == 0) pol.seg_meta(seg);
+        flush(EndSlot{seg, s_cur >= 0 ? 0 : -1}, false);
     }
 }
 
