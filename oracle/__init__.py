@@ -24,7 +24,7 @@ from dataclasses import dataclass
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = os.path.join(_HERE, "tbe_oracle.cpp")
+_SRCS = [os.path.join(_HERE, "tbe_oracle.cpp"), os.path.join(_HERE, "fm_oracle.cpp")]
 _LIB = os.path.join(_HERE, "libtbe_oracle.so")
 
 # Storage codes understood by the C++ file.
@@ -45,11 +45,11 @@ class OracleError(RuntimeError):
 def build(force: bool = False) -> str:
     """Compile the oracle with g++ (OpenMP, no FMA contraction) if it is stale."""
     if (not force and os.path.exists(_LIB)
-            and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
+            and all(os.path.getmtime(_LIB) >= os.path.getmtime(s) for s in _SRCS)):
         return _LIB
     tmp = _LIB + f".tmp{os.getpid()}"
     cmd = ["g++", "-std=c++17", "-O2", "-ffp-contract=off", "-fopenmp", "-shared", "-fPIC",
-           _SRC, "-o", tmp]
+           *_SRCS, "-o", tmp]
     subprocess.run(cmd, check=True)
     os.replace(tmp, _LIB)
     return _LIB
@@ -82,6 +82,10 @@ def _load():
         lib.tbe_oracle_backward_free.restype = None
         lib.tbe_oracle_backward_dense.argtypes = [i32, p, p, i32, p, i32, i64, p, p, i32, p, p]
         lib.tbe_oracle_backward_dense.restype = ctypes.c_int
+        lib.fm_oracle_forward.argtypes = [i32, i32, i32, i64, p, p]
+        lib.fm_oracle_forward.restype = ctypes.c_int
+        lib.fm_oracle_backward.argtypes = [i32, i32, i32, i64, p, p, p]
+        lib.fm_oracle_backward.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -226,3 +230,35 @@ def backward_dense(rows, dims, batch: int, indices, offsets, grad_out, weights=N
     if st != OK:
         raise OracleError(st)
     return dense
+
+
+# ----------------------------------------------------------------------------- FM cross term
+
+def _fm_input(y, num_fields: int):
+    y = _np(y, np.float32)
+    if y.ndim != 2 or num_fields <= 0 or y.shape[1] % num_fields:
+        raise ValueError("y must be [B, T * D] with T = num_fields")
+    return y, y.shape[0], y.shape[1] // num_fields
+
+
+def fm_forward(y, num_fields: int, threads: int = 0) -> np.ndarray:
+    """fm[b] = sum over field pairs t < u of <v_bt, v_bu> in float64 (fm_oracle.cpp)."""
+    y, B, D = _fm_input(y, num_fields)
+    out = np.zeros(B, dtype=np.float64)
+    st = _load().fm_oracle_forward(B, num_fields, D, y.shape[1], _ptr(y), _ptr(out))
+    if st != OK:
+        raise OracleError(st)
+    return out
+
+
+def fm_backward(y, grad_fm, num_fields: int) -> np.ndarray:
+    """grad_y[b, t*D + j] = g[b] * sum over u != t of y[b, u*D + j], float64 [B, T*D]."""
+    y, B, D = _fm_input(y, num_fields)
+    g = _np(grad_fm, np.float32)
+    if g.shape != (B,):
+        raise ValueError("grad_fm must be [B]")
+    out = np.zeros((B, num_fields * D), dtype=np.float64)
+    st = _load().fm_oracle_backward(B, num_fields, D, y.shape[1], _ptr(y), _ptr(g), _ptr(out))
+    if st != OK:
+        raise OracleError(st)
+    return out
