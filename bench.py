@@ -389,6 +389,9 @@ def run_ours(args):
     # The reuse-free control: the forward over uniform indices on the same tables.
     if w.zipf_alpha is not None and not args.no_control:
         line["control_uniform"] = run_control(args, m, w, dev, out, flush, world, peak)
+    # Next rows on the same pooled output: the FM cross term and its gradient.
+    if not args.no_next and len(set(w.dims)) == 1:
+        line["next_rows"] = {"fm": run_fm(w, out, flush, dev, peak)}
     # End to end through the public API from pinned host memory.
     if not args.no_e2e:
         line["e2e"] = run_e2e(args, m, w, batches, grads_out, g, out, dev, world)
@@ -436,6 +439,44 @@ def run_control(args, m, w, dev, out, flush, world, peak):
     if traffic:
         res["gather_frac_dram"] = round(traffic / (gms * 1e-3) / 1e9 / peak, 4)
     del batches
+    return res
+
+
+def run_fm(w, y, flush, dev, peak):
+    """FM cross term (cb_fm_forward) and its gradient (cb_fm_backward) on the pooled
+    output of the last forward: fields = tables, inputs larger than L2."""
+    from paper_2609_30656_gb300 import tbe
+    T, D, B = w.num_tables, w.dims[0], w.batch
+    g = torch.Generator(device=dev)
+    g.manual_seed(11)
+    grad_fm = torch.randn(B, generator=g, device=dev)
+    fm = torch.empty(B, dtype=torch.float32, device=dev)
+    grad_y = torch.empty_like(y)
+    res = {}
+    for name, backward in (("forward", False), ("backward", True)):
+        def call():
+            if backward:
+                tbe.fm_backward(y, grad_fm, T, out=grad_y)
+            else:
+                tbe.fm_forward(y, T, out=fm)
+        for _ in range(2):
+            call()
+        torch.cuda.synchronize()
+        reps = 5
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for a, b in ev:
+            flush.zero_()
+            a.record()
+            call()
+            b.record()
+        torch.cuda.synchronize()
+        ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+        nbytes = metrics.fm_bytes(B, T, D, backward)
+        res[name] = {"ms": round(ms, 4), "alg_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
+                     "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes}
+    res["shape"] = f"{B} samples x {T} fields x dim {D} (fp32 pooled rows)"
+    del grad_y
     return res
 
 
@@ -567,6 +608,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-control", action="store_true",
                     help="skip the forward on uniform indices over the same tables")
+    ap.add_argument("--no-next", action="store_true",
+                    help="skip the next-row measurements (FM cross term)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
     if args.impl == "reference":

@@ -181,6 +181,38 @@ const char* cb_tbe_status_string(cb_status s);
 /* Releases the workspace and the handle (synchronises its last stream). */
 void cb_tbe_destroy(cb_tbe* h);
 
+/* ---------------------------------------------------------------------------
+ * Factorization-machine cross term on the pooled rows: the inter_arch.fm step
+ * that follows the lookups in the paper's DeepFM-based model (Sec. IV.A.2,
+ * bandwidth-bound element-wise and reduction passes). Each of the T fields is
+ * one table's pooled row, all of one dim D: v_bt = y[b, t*D : (t+1)*D], and
+ *
+ *   fm[b] = sum_{t < u} <v_bt, v_bu>          (Rendle's second-order term)
+ *   grad_y[b, t*D + j] = grad_fm[b] * sum_{u != t} y[b, u*D + j]
+ *
+ * The sums are taken in fp32 in a fixed order (deterministic). These calls
+ * need no handle and allocate nothing.
+ *   y           device fp32 [batch, row_stride], 16-byte aligned; field t of
+ *               sample b at y + b*row_stride + t*dim (the output of
+ *               cb_tbe_forward over T tables of dim D, row_stride = T*D)
+ *   batch       >= 0 samples
+ *   num_fields  T >= 1
+ *   dim         D, a multiple of 4, 4 <= D <= 512
+ *   row_stride  floats from one sample to the next, >= T*D, a multiple of 4
+ * Invalid arguments return CB_ERR_INVALID_ARG before any GPU work; a failed
+ * launch returns CB_ERR_CUDA. */
+
+/* out: device fp32 [batch], fm[b]. */
+cb_status cb_fm_forward(const float* y, int32_t batch, int32_t num_fields, int32_t dim,
+                        int64_t row_stride, float* out, cudaStream_t stream);
+
+/* grad_fm: device fp32 [batch]; grad_y: device fp32, the layout of y (16-byte
+ * aligned); columns [0, T*D) of every row are written, the rest untouched.
+ * grad_y may be passed to cb_tbe_backward as its grad_out when
+ * row_stride = T*D. */
+cb_status cb_fm_backward(const float* y, const float* grad_fm, int32_t batch, int32_t num_fields,
+                         int32_t dim, int64_t row_stride, float* grad_y, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

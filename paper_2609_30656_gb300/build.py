@@ -20,7 +20,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcb_tbe.so")
 SOURCES = ["cb_tbe.cu", "tbe_plan.cu", "tbe_forward.cu", "tbe_forward_f32.cu", "tbe_forward_f16.cu",
-           "tbe_forward_bf16.cu", "tbe_backward.cu", "tbe_sort.cu", "cb_tbe_noalloc.cu"]
+           "tbe_forward_bf16.cu", "tbe_backward.cu", "tbe_sort.cu", "cb_tbe_noalloc.cu",
+           "fm_interaction.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -110,3 +110,10 @@ def component_bytes(c: BatchCounts, unique_per_table, rows, packed: bool) -> dic
         "bwd.reduce": b["grad_gather"] + 4 * n + (8 * n if packed else 0) + 4 * U + b["grads"]
         + 16 * U,
     }
+
+
+def fm_bytes(batch: int, num_fields: int, dim: int, backward: bool) -> int:
+    """Algorithmic bytes of the FM cross term: the pooled rows read once (fp32),
+    plus fm [B] written (forward), or grad_fm [B] read and grad_y written (backward)."""
+    y = 4 * batch * num_fields * dim
+    return y + 4 * batch + (y if backward else 0)

@@ -29,7 +29,7 @@ _IDX = {torch.int32: 0, torch.int64: 1}
 EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
-           "cb_tbe_forward_noalloc")
+           "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -78,8 +78,10 @@ def load_library() -> ctypes.CDLL:
     lib.cb_tbe_status_string.restype = ctypes.c_char_p
     lib.cb_tbe_destroy.argtypes = [p]
     lib.cb_tbe_destroy.restype = None
+    lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
+    lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
-                 "cb_tbe_get_error", "cb_tbe_last_timings"):
+                 "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -268,3 +270,45 @@ class TBE:
 
     def launch_count(self) -> int:
         return int(self._lib.cb_tbe_launch_count(self._h))
+
+
+# ----------------------------------------------------------------------------- FM cross term
+
+def _fm_args(y: torch.Tensor, num_fields: int):
+    if y.device.type != "cuda" or y.dtype != torch.float32 or y.dim() != 2:
+        raise ValueError("y must be a 2-D fp32 CUDA tensor [B, T * D]")
+    if y.stride(1) != 1:
+        raise ValueError("y rows must be contiguous")
+    if num_fields < 1 or y.shape[1] % num_fields:
+        raise ValueError("the row length must be num_fields * dim")
+    return y.shape[0], y.shape[1] // num_fields, y.stride(0)
+
+
+def fm_forward(y: torch.Tensor, num_fields: int, out: torch.Tensor | None = None) -> torch.Tensor:
+    """fm[b] = sum over field pairs t < u of <y[b, tD:(t+1)D], y[b, uD:(u+1)D]> (cb_fm_forward)."""
+    lib = load_library()
+    B, D, stride = _fm_args(y, num_fields)
+    if out is None:
+        out = torch.empty(B, dtype=torch.float32, device=y.device)
+    with torch.cuda.device(y.device):
+        stream = ctypes.c_void_p(torch.cuda.current_stream(y.device).cuda_stream)
+        _check(lib.cb_fm_forward(_ptr(y), B, num_fields, D, stride, _ptr(out), stream),
+               "cb_fm_forward")
+    return out
+
+
+def fm_backward(y: torch.Tensor, grad_fm: torch.Tensor, num_fields: int,
+                out: torch.Tensor | None = None) -> torch.Tensor:
+    """grad_y[b, tD + j] = grad_fm[b] * sum over u != t of y[b, uD + j] (cb_fm_backward)."""
+    lib = load_library()
+    B, D, stride = _fm_args(y, num_fields)
+    if grad_fm.device != y.device or grad_fm.dtype != torch.float32 or grad_fm.numel() != B:
+        raise ValueError("grad_fm must be fp32 [B] on the device of y")
+    grad_fm = grad_fm.contiguous()
+    if out is None:
+        out = torch.empty_strided(y.shape, y.stride(), dtype=torch.float32, device=y.device)
+    with torch.cuda.device(y.device):
+        stream = ctypes.c_void_p(torch.cuda.current_stream(y.device).cuda_stream)
+        _check(lib.cb_fm_backward(_ptr(y), _ptr(grad_fm), B, num_fields, D, stride, _ptr(out),
+                                  stream), "cb_fm_backward")
+    return out

@@ -13,7 +13,7 @@ def _declared_functions():
     with open(os.path.join(ROOT, "include", "cb_tbe.h")) as f:
         text = f.read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(cb_tbe_\w+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(cb_(?:tbe|fm)_\w+)\s*\(", text)))
 
 
 @pytest.fixture(scope="module")
@@ -67,6 +67,12 @@ def test_host_side_argument_errors_return_before_any_gpu_work(lib):
     assert lib.cb_tbe_reserve(None, 1, 1) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_tbe_launch_count(None) == 0
     lib.cb_tbe_destroy(None)
+    # the FM cross term: null buffers, a dim that is not a multiple of 4, no fields
+    assert lib.cb_fm_forward(None, 1, 2, 8, 16, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_fm_forward(None, 0, 2, 6, 12, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_fm_backward(None, None, 0, 0, 8, 0, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_fm_backward(None, None, 4, 2, 8, 12, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_fm_forward(None, 0, 2, 8, 16, None, None) == tbe.CB_OK  # nothing to do
 
 
 def test_product_path_fails_loudly_without_the_library(monkeypatch, tmp_path):

@@ -27,6 +27,12 @@ def test_forward_and_backward_bytes_by_hand():
     assert metrics.forward_unique_bytes(c, [3, 1]) == f["total"] - f["rows"] + 3 * 8 + 1 * 16
 
 
+def test_fm_bytes_by_hand():
+    # 3 samples x 2 fields x dim 4: 24 floats of pooled rows
+    assert metrics.fm_bytes(3, 2, 4, backward=False) == 24 * 4 + 3 * 4
+    assert metrics.fm_bytes(3, 2, 4, backward=True) == 2 * 24 * 4 + 3 * 4
+
+
 def test_radix_passes_follow_row_bits():
     assert metrics.radix_passes([256]) == 1
     assert metrics.radix_passes([257]) == 2
