@@ -480,6 +480,31 @@ def run_fm(w, y, flush, dev, peak):
     return res
 
 
+def run_fm_only(args):
+    """The FM cross term alone on y ~ N(0, 0.05^2) of shape [batch, T * D]."""
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = workload_of(args)
+    if len(set(w.dims)) != 1:
+        raise SystemExit("the FM cross term needs tables of one dim")
+    g = torch.Generator(device=dev)
+    g.manual_seed(args.seed)
+    y = torch.randn(w.batch, w.sum_dims, generator=g, device=dev).mul_(0.05)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev)
+    peak, _ = measured_hbm_peak()
+    with ClockSampler(0) as clk:
+        res = run_fm(w, y, flush, dev, peak)
+    ms = res["forward"]["ms"] + res["backward"]["ms"]
+    nbytes = res["forward"]["bytes"] + res["backward"]["bytes"]
+    print(json.dumps({
+        "metric": "FM cross term forward + backward, algorithmic HBM GB/s", "unit": "GB/s",
+        "value": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms_per_step": round(ms, 4), "n_gpus": 1,
+        "higher_is_better": True, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": res["shape"]}, "next_rows": {"fm": res}, "clocks": clk.summary()}),
+        flush=True)
+
+
 def run_e2e(args, m, w, batches, grads_out, g, out, dev, world):
     b, go = batches[0], grads_out[0]
     h_ind = b.indices.cpu().pin_memory()
@@ -610,10 +635,15 @@ def main(argv=None):
                     help="skip the forward on uniform indices over the same tables")
     ap.add_argument("--no-next", action="store_true",
                     help="skip the next-row measurements (FM cross term)")
+    ap.add_argument("--fm-only", action="store_true",
+                    help="time only the FM cross term and its gradient on a synthetic pooled "
+                         "output of the workload's shape (no tables are allocated)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
     if args.impl == "reference":
         run_reference(args)
+    elif args.fm_only:
+        run_fm_only(args)
     else:
         run_ours(args)
 

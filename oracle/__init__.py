@@ -82,6 +82,8 @@ def _load():
         lib.tbe_oracle_backward_free.restype = None
         lib.tbe_oracle_backward_dense.argtypes = [i32, p, p, i32, p, i32, i64, p, p, i32, p, p]
         lib.tbe_oracle_backward_dense.restype = ctypes.c_int
+        lib.tbe_oracle_weight_grad.argtypes = [i32, p, p, p, p, i32, p, i32, i64, p, i32, p, i32, p]
+        lib.tbe_oracle_weight_grad.restype = ctypes.c_int
         lib.fm_oracle_forward.argtypes = [i32, i32, i32, i64, p, p]
         lib.fm_oracle_forward.restype = ctypes.c_int
         lib.fm_oracle_backward.argtypes = [i32, i32, i32, i64, p, p, p]
@@ -163,6 +165,27 @@ def forward(tables, batch: int, indices, offsets, weights=None, mean: bool = Fal
     st = _load().tbe_oracle_forward(T, _ptr(rows), _ptr(dims), _ptr(codes),
                                     ctypes.cast(ptrs, ctypes.c_void_p), batch, _ptr(ind), is32,
                                     ind.shape[0], _ptr(off), _ptr(w), int(mean), threads, _ptr(out))
+    if st != OK:
+        raise OracleError(st)
+    return out
+
+
+def weight_grad(tables, batch: int, indices, offsets, grad_out, mean: bool = False,
+                threads: int = 0) -> np.ndarray:
+    """d<grad_out, y>/d w_i = s_b * <grad_out[b, Doff_t:], E_t[idx_i]>, float64 [n]."""
+    arrs = [_table_array(t) for t in tables]
+    T = len(arrs)
+    rows = np.array([a.shape[0] for a, _ in arrs], dtype=np.int64)
+    dims = np.array([a.shape[1] for a, _ in arrs], dtype=np.int32)
+    codes = np.array([c for _, c in arrs], dtype=np.int32)
+    ptrs = (ctypes.c_void_p * T)(*[a.ctypes.data for a, _ in arrs])
+    ind, off, is32 = _index_arrays(indices, offsets)
+    go = _np(grad_out, np.float32)
+    out = np.zeros(ind.shape[0], dtype=np.float64)
+    st = _load().tbe_oracle_weight_grad(T, _ptr(rows), _ptr(dims), _ptr(codes),
+                                        ctypes.cast(ptrs, ctypes.c_void_p), batch, _ptr(ind), is32,
+                                        ind.shape[0], _ptr(off), int(mean), _ptr(go), threads,
+                                        _ptr(out))
     if st != OK:
         raise OracleError(st)
     return out

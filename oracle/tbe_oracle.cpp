@@ -190,6 +190,46 @@ int tbe_oracle_forward(int32_t T, const int64_t* rows, const int32_t* dims, cons
     return ORC_OK;
 }
 
+// Gradient with respect to the per-sample weights. The output is linear in
+// each w_i, so d<grad_out, y>/d w_i = s_b * sum_j grad_out[b, Doff_t + j] *
+// E_t[indices[i], j] (s_b = 1/L for mean pooling, 1 for sum), whatever the
+// weights are; out is [n] in lookup order.
+int tbe_oracle_weight_grad(int32_t T, const int64_t* rows, const int32_t* dims, const int32_t* dtypes,
+                           const void* const* tables, int32_t B, const void* indices,
+                           int32_t idx_is_i32, int64_t n, const void* offsets, int32_t mean_pooling,
+                           const float* grad_out, int32_t threads, double* out) {
+    int st = check_common(T, rows, dims, B, n, indices, offsets, idx_is_i32);
+    if (st != ORC_OK) return st;
+    if ((n > 0 && !out) || !dtypes || !tables || (n > 0 && B > 0 && !grad_out)) return ORC_BAD_ARG;
+
+    std::vector<int64_t> doff(T + 1, 0);
+    for (int32_t t = 0; t < T; ++t) doff[t + 1] = doff[t] + dims[t];
+    const int64_t sum_d = doff[T];
+    const int64_t num_bags = static_cast<int64_t>(T) * B;
+
+#ifdef _OPENMP
+    const int nthr = threads > 0 ? threads : omp_get_max_threads();
+#pragma omp parallel for schedule(dynamic, 16) num_threads(nthr)
+#endif
+    for (int64_t bag = 0; bag < num_bags; ++bag) {
+        const int32_t t = static_cast<int32_t>(bag / B);
+        const int64_t b = bag % B;
+        const int32_t D = dims[t];
+        const int64_t s = read_index(offsets, idx_is_i32, bag);
+        const int64_t e = read_index(offsets, idx_is_i32, bag + 1);
+        const double scale = mean_pooling && e > s ? 1.0 / static_cast<double>(e - s) : 1.0;
+        const float* g = grad_out + b * sum_d + doff[t];
+        for (int64_t i = s; i < e; ++i) {
+            const int64_t r = read_index(indices, idx_is_i32, i);
+            double dot = 0.0;
+            for (int32_t j = 0; j < D; ++j)
+                dot += static_cast<double>(g[j]) * table_value(tables[t], dtypes[t], r * D + j);
+            out[i] = scale * dot;
+        }
+    }
+    return ORC_OK;
+}
+
 // Backward, de-duplicated: stable comparison sort of (key, position) by key,
 // runs of equal keys, then one fp64 sum per run in ascending position order.
 // The result is held in an opaque object; fetch it with the calls below.

@@ -289,3 +289,46 @@ def test_malformed_offsets_are_an_error(mutate):
     rows, dims = table_meta(tables)
     with pytest.raises(oracle.OracleError):
         oracle.backward(rows, dims, 9, ind, off2, torch.zeros(9, int(dims.sum())))
+
+
+# ---------------------------------------------------------------- weight gradient
+
+@pytest.mark.parametrize("case", ["sum", "mean"])
+def test_weight_grad_hand_worked(golden, case):
+    g, tables, ind, off, _, go = _golden_problem(golden)
+    got = oracle.weight_grad(tables, g["batch"], ind, off, go, mean=case == "mean")
+    want = np.array([parse_value(v) for v in g["weight_grad"][case]])
+    np.testing.assert_allclose(got, want, rtol=1e-15, atol=0)
+
+
+@pytest.mark.parametrize("mean", [False, True])
+def test_weight_grad_matches_torch_autograd(mean):
+    tables, ind, off, w = random_problem(41, weighted=True, max_len=30)
+    rows, dims = table_meta(tables)
+    go = torch.randn(9, int(dims.sum()), generator=torch.Generator().manual_seed(4),
+                     dtype=torch.float32)
+    wl_ = w.to(torch.float64).clone().requires_grad_(True)
+    y = torch_forward_f64(tables, 9, ind, off, wl_, mean)
+    (y * go.to(torch.float64)).sum().backward()
+    got = oracle.weight_grad(tables, 9, ind, off, go, mean=mean)
+    np.testing.assert_allclose(got, wl_.grad.numpy(), rtol=1e-12, atol=1e-13)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_weight_grad_adjoint_identity_and_exact_differences(dtype):
+    # y is linear in the weights: <grad_out, y(w)> = sum_i w_i * grad_w_i, and
+    # with integer data y(w + e_i) - y(w) gives grad_w_i exactly.
+    tables, ind, off, w = random_problem(42, dtype=dtype, int_valued=True, weighted=True,
+                                         max_len=20)
+    rows, dims = table_meta(tables)
+    go = torch.randint(-8, 9, (9, int(dims.sum())),
+                       generator=torch.Generator().manual_seed(5)).to(torch.float32)
+    gw = oracle.weight_grad(tables, 9, ind, off, go)
+    y = oracle.forward(tables, 9, ind, off, weights=w)
+    gd = go.double().numpy()
+    assert (gd * y).sum() == (w.double().numpy() * gw).sum()
+    for i in range(0, ind.numel(), max(1, ind.numel() // 25)):
+        w2 = w.clone()
+        w2[i] += 1.0
+        dy = oracle.forward(tables, 9, ind, off, weights=w2) - y
+        assert (gd * dy).sum() == gw[i]
