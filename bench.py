@@ -389,9 +389,14 @@ def run_ours(args):
     # The reuse-free control: the forward over uniform indices on the same tables.
     if w.zipf_alpha is not None and not args.no_control:
         line["control_uniform"] = run_control(args, m, w, dev, out, flush, world, peak)
-    # Next rows on the same pooled output: the FM cross term and its gradient.
-    if not args.no_next and len(set(w.dims)) == 1:
-        line["next_rows"] = {"fm": run_fm(w, out, flush, dev, peak)}
+    # Next rows: the FM cross term and its gradient on the same pooled output,
+    # and the gradient of the per-sample weights on the first batch.
+    if not args.no_next:
+        nxt = {}
+        if len(set(w.dims)) == 1:
+            nxt["fm"] = run_fm(w, out, flush, dev, peak)
+        nxt["weight_grad"] = run_weight_grad(m, batches[0], grads_out[0], counts[0], flush, peak)
+        line["next_rows"] = nxt
     # End to end through the public API from pinned host memory.
     if not args.no_e2e:
         line["e2e"] = run_e2e(args, m, w, batches, grads_out, g, out, dev, world)
@@ -478,6 +483,32 @@ def run_fm(w, y, flush, dev, peak):
     res["shape"] = f"{B} samples x {T} fields x dim {D} (fp32 pooled rows)"
     del grad_y
     return res
+
+
+def run_weight_grad(m, b, go, c, flush, peak):
+    """d<grad_out, y>/d w for every lookup (cb_tbe_weight_grad) on one batch."""
+    gw = torch.empty(b.num_indices, dtype=torch.float32, device=go.device)
+    for _ in range(2):
+        m.weight_grad(b.indices, b.offsets, go, out=gw)
+    torch.cuda.synchronize()
+    reps = 5
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps)]
+    for a, e in ev:
+        flush.zero_()
+        a.record()
+        m.weight_grad(b.indices, b.offsets, go, out=gw)
+        e.record()
+    torch.cuda.synchronize()
+    if m.get_error() != 0:
+        raise RuntimeError("device-side error in the weight gradient")
+    ms = statistics.mean(a.elapsed_time(e) for a, e in ev)
+    nbytes = metrics.weight_grad_bytes(c)
+    del gw
+    return {"ms": round(ms, 4), "alg_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
+            "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes,
+            "note": "algorithmic bytes count each lookup's row and grad_out slice; "
+                    "repeated rows and a table's grad_out slice are largely served by L2"}
 
 
 def run_fm_only(args):

@@ -178,6 +178,18 @@ uint64_t cb_tbe_launch_count(const cb_tbe* h);
 /* Short English description of a status code. */
 const char* cb_tbe_status_string(cb_status s);
 
+/* Gradient with respect to the per-sample weights (not in the paper; the
+ * pooled bag above is linear in each weight, so this is its exact derivative):
+ *   grad_weights[i] = s_b * sum_j grad_out[b, Doff_t + j] * E_t[indices[i], j]
+ * for lookup i of bag (t, b), s_b = 1/L (mean pooling) or 1 (sum). The weights
+ * themselves are not needed. Same batch, indices, num_indices and offsets as
+ * cb_tbe_forward; grad_out device fp32 [B, sum of dims], 16-byte aligned;
+ * grad_weights device fp32 [num_indices], every element written (0 for an
+ * out-of-range index, which also sets CB_ERR_INDEX_OOB). Deterministic. */
+cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                             const void* offsets, const float* grad_out, float* grad_weights,
+                             cudaStream_t stream);
+
 /* Releases the workspace and the handle (synchronises its last stream). */
 void cb_tbe_destroy(cb_tbe* h);
 

@@ -488,6 +488,41 @@ cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t 
     return finish_call(h, stream);
 }
 
+cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                             const void* offsets, const float* grad_out, float* grad_weights,
+                             cudaStream_t stream) {
+    cb_status st = check_common(h, batch, indices, num_indices, offsets);
+    if (st != CB_OK) return st;
+    const int64_t n = num_indices;
+    if (n > 0 && batch > 0 &&
+        (!grad_out || !grad_weights || (reinterpret_cast<uintptr_t>(grad_out) & 15u)))
+        return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    h->last_stream = stream;
+    if (n == 0 || batch == 0) return CB_OK;
+    Problem P = make_problem(h, batch, indices, n, offsets, nullptr);
+    if (h->flags & CB_VALIDATE) {
+        launch_validate_offsets(P, h->num_sms, stream);
+        h->launches += 1;
+    }
+    st = ensure_workspace(h, batch, n);
+    if (st != CB_OK) return st;
+    Workspace w;
+    layout(h, batch, n, static_cast<char*>(h->ws), &w);
+    Plan Q = make_plan(h, w, false, kFwdChunk);
+    const int64_t bound = n / kFwdChunk + h->T + 1;
+    launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
+    h->launches += 2;
+    for (size_t c = 0; c < h->fwd_classes.size(); ++c) {
+        // The compiled row layouts cover one vector per lane; wider rows loop.
+        const int gc = h->fwd_classes[c].vpl == 1 ? h->fwd_classes[c].gc : 0;
+        launch_weight_grad(P, Q, grad_out, grad_weights, static_cast<int>(c), h->fwd_classes[c].dtype, gc,
+                           bound, h->num_sms, stream);
+        h->launches += 1;
+    }
+    return finish_call(h, stream);
+}
+
 cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
                           const void* offsets, const float* per_sample_weights,
                           const float* grad_out, cb_sparse_grad* g, cudaStream_t stream) {

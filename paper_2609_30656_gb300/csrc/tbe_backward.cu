@@ -31,34 +31,12 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
         const TableDev& td = P.tables[t];
         const int64_t k0 = ch.k0, k1 = ch.k0 + (ch.len & 0x7fffffffu);
         const int64_t bag_lo = static_cast<int64_t>(t) * P.B, bag_hi = bag_lo + P.B;
-        // Window of 32 bag ends: lane i holds the end of bag win + i.
-        int64_t win = ch.first;
-        int64_t win_start = win < bag_hi ? load_index(P.offsets, win, P.is32) : kNoSeg;
-        int64_t my_end = (win + lane < bag_hi) ? load_index(P.offsets, win + lane + 1, P.is32) : kNoSeg;
+        BagWindow W = bag_window(P, ch.first, bag_hi, lane);
         for (int64_t base = k0; base < k1; base += 32) {
             const int64_t q = base + lane;
             const bool valid = q < k1;
-            int64_t my_bag = -1, my_s = 0, my_e = 0;
-            while (true) {
-                // Ends in the window never decrease (valid offsets), so the number
-                // of bags of the window that end at or before q is a binary search.
-                int cnt = 0;
-#pragma unroll
-                for (int b = 16; b >= 1; b >>= 1)
-                    if (__shfl_sync(kFull, my_end, cnt + b - 1) <= q) cnt += b;
-                if (__shfl_sync(kFull, my_end, 31) <= q) cnt = 32;
-                const int64_t e_sel = __shfl_sync(kFull, my_end, cnt < 32 ? cnt : 31);
-                const int64_t s_sel = __shfl_sync(kFull, my_end, cnt > 0 ? cnt - 1 : 0);
-                if (valid && my_bag < 0 && cnt < 32) {
-                    my_bag = win + cnt;
-                    my_e = e_sel;
-                    my_s = cnt > 0 ? s_sel : win_start;
-                }
-                if (!__any_sync(kFull, valid && my_bag < 0)) break;
-                win_start = __shfl_sync(kFull, my_end, 31);
-                win += 32;
-                my_end = (win + lane < bag_hi) ? load_index(P.offsets, win + lane + 1, P.is32) : kNoSeg;
-            }
+            int64_t my_bag, my_s, my_e;
+            find_bag(P, W, q, valid, lane, my_bag, my_s, my_e);
             if (valid) {
                 if (my_bag >= bag_hi) {  // only reachable with malformed offsets
                     set_error(P.error, CB_ERR_BAD_OFFSETS);

@@ -136,6 +136,56 @@ __device__ __forceinline__ int64_t warps_in_grid() {
     return (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
 }
 
+// ---------------------------------------------------------------- bags of positions
+
+// The bag of each of 32 consecutive lookup positions of one table. A window of
+// 32 bag ends slides forward (lane i holds the end of bag win + i); ends never
+// decrease (valid offsets), so the number of the window's bags that end at or
+// before a position is a bisection. Each lane gets its bag and the bag's
+// [start, end) positions.
+struct BagWindow {
+    int64_t win;        // first bag of the window
+    int64_t win_start;  // start position of bag win
+    int64_t my_end;     // end position of bag win + lane (kNoSeg past the table)
+    int64_t bag_hi;     // one past the table's last bag
+};
+
+__device__ __forceinline__ BagWindow bag_window(const Problem& P, int64_t first, int64_t bag_hi,
+                                                int lane) {
+    BagWindow W;
+    W.win = first;
+    W.bag_hi = bag_hi;
+    W.win_start = first < bag_hi ? load_index(P.offsets, first, P.is32) : kNoSeg;
+    W.my_end = (first + lane < bag_hi) ? load_index(P.offsets, first + lane + 1, P.is32) : kNoSeg;
+    return W;
+}
+
+// Every lane of the warp calls this with its position q (valid: q is a lookup
+// of the table); bag = -1 for invalid lanes.
+__device__ __forceinline__ void find_bag(const Problem& P, BagWindow& W, int64_t q, bool valid, int lane,
+                                         int64_t& bag, int64_t& s, int64_t& e) {
+    bag = -1;
+    s = e = 0;
+    while (true) {
+        int cnt = 0;
+#pragma unroll
+        for (int b = 16; b >= 1; b >>= 1)
+            if (__shfl_sync(kFull, W.my_end, cnt + b - 1) <= q) cnt += b;
+        if (__shfl_sync(kFull, W.my_end, 31) <= q) cnt = 32;
+        const int64_t e_sel = __shfl_sync(kFull, W.my_end, cnt < 32 ? cnt : 31);
+        const int64_t s_sel = __shfl_sync(kFull, W.my_end, cnt > 0 ? cnt - 1 : 0);
+        if (valid && bag < 0 && cnt < 32) {
+            bag = W.win + cnt;
+            e = e_sel;
+            s = cnt > 0 ? s_sel : W.win_start;
+        }
+        if (!__any_sync(kFull, valid && bag < 0)) break;
+        W.win_start = __shfl_sync(kFull, W.my_end, 31);
+        W.win += 32;
+        W.my_end = (W.win + lane < W.bag_hi) ? load_index(P.offsets, W.win + lane + 1, P.is32) : kNoSeg;
+    }
+}
+
 // ---------------------------------------------------------------- storage types
 
 template <int DT> struct Storage;

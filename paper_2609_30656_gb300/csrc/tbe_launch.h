@@ -95,6 +95,8 @@ inline int compile_time_groups(int vpl, int lanes, int groups) {
     if (lanes * groups == 32 && (groups == 1 || groups == 2 || groups == 4 || groups == 8)) return groups;
     return 0;
 }
+void launch_weight_grad(const Problem& P, const Plan& Q, const float* grad_out, float* grad_w, int cls,
+                        int dtype, int gc, int64_t chunk_bound, int num_sms, cudaStream_t s);
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
 

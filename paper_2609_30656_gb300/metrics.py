@@ -11,6 +11,10 @@ result table (Sec. IV.A.1) divided by the achieved time gives the same
   backward  per lookup: D_t * 4 (gathered grad_out slice) + idx_bytes (+ 4)
             per bag:    idx_bytes              per unique row: 8 (id) + D_t * 4
   sort      per lookup and pass: 16 (read and write a 4-byte key and payload)
+  weight gradient  per lookup: D_t * e_S (stored row) + D_t * 4 (grad_out slice)
+            + idx_bytes + 4 (the gradient)    per bag: idx_bytes
+  FM cross term    per pooled value: 4 read (+ 4 written by the backward);
+            per sample: 4 (fm written, or grad_fm read)
 """
 
 from __future__ import annotations
@@ -80,6 +84,13 @@ def backward_bytes(c: BatchCounts, unique_per_table) -> dict[str, int]:
     }
     parts["total"] = sum(parts.values())
     return parts
+
+
+def weight_grad_bytes(c: BatchCounts) -> int:
+    """Algorithmic bytes of d<grad_out, y>/d w: each lookup's row and grad_out slice."""
+    rows = sum(L * d * c.elem_bytes for L, d in zip(c.lookups_per_table, c.dims))
+    slices = sum(L * d * 4 for L, d in zip(c.lookups_per_table, c.dims))
+    return rows + slices + c.n * (c.idx_bytes + 4) + (c.num_tables * c.batch + 1) * c.idx_bytes
 
 
 def sort_bytes(n: int, passes: int) -> int:

@@ -29,7 +29,7 @@ _IDX = {torch.int32: 0, torch.int64: 1}
 EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
-           "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward")
+           "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -78,10 +78,12 @@ def load_library() -> ctypes.CDLL:
     lib.cb_tbe_status_string.restype = ctypes.c_char_p
     lib.cb_tbe_destroy.argtypes = [p]
     lib.cb_tbe_destroy.restype = None
+    lib.cb_tbe_weight_grad.argtypes = [p, i32, p, i64, p, p, p, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
-                 "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward"):
+                 "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward",
+                 "cb_tbe_weight_grad"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -251,6 +253,22 @@ class TBE:
         U, F = probe.num_unique, probe.num_floats
         g = self.alloc_grad(U, F)
         return self.backward_into(g, indices, offsets, grad_out, per_sample_weights)
+
+    def weight_grad(self, indices, offsets, grad_out,
+                    out: torch.Tensor | None = None) -> torch.Tensor:
+        """d<grad_out, y>/d w_i for every lookup i (cb_tbe_weight_grad), fp32 [n]."""
+        T = len(self.dims)
+        batch = (offsets.numel() - 1) // T
+        ind = self._dev(indices, self.index_dtype)
+        off = self._dev(offsets, self.index_dtype)
+        go = self._dev(grad_out, torch.float32)
+        if out is None:
+            out = torch.empty(ind.numel(), dtype=torch.float32, device=self.device)
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_weight_grad(self._h, batch, _ptr(ind), ind.numel(), _ptr(off),
+                                                _ptr(go), _ptr(out), self._stream()),
+                   "cb_tbe_weight_grad")
+        return out
 
     def get_error(self) -> int:
         with torch.cuda.device(self.device):

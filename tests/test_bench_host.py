@@ -27,6 +27,15 @@ def test_forward_and_backward_bytes_by_hand():
     assert metrics.forward_unique_bytes(c, [3, 1]) == f["total"] - f["rows"] + 3 * 8 + 1 * 16
 
 
+def test_weight_grad_bytes_by_hand():
+    # 2 tables (dims 4 and 8, fp16), batch 3, lookups 5 and 2
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts((4, 8), 2, 3, off, weighted=False)
+    rows = 5 * 4 * 2 + 2 * 8 * 2
+    slices = 5 * 4 * 4 + 2 * 8 * 4
+    assert metrics.weight_grad_bytes(c) == rows + slices + 7 * (8 + 4) + 7 * 8
+
+
 def test_fm_bytes_by_hand():
     # 3 samples x 2 fields x dim 4: 24 floats of pooled rows
     assert metrics.fm_bytes(3, 2, 4, backward=False) == 24 * 4 + 3 * 4
