@@ -24,7 +24,8 @@ from dataclasses import dataclass
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRCS = [os.path.join(_HERE, "tbe_oracle.cpp"), os.path.join(_HERE, "fm_oracle.cpp")]
+_SRCS = [os.path.join(_HERE, "tbe_oracle.cpp"), os.path.join(_HERE, "fm_oracle.cpp"),
+         os.path.join(_HERE, "opt_oracle.cpp")]
 _LIB = os.path.join(_HERE, "libtbe_oracle.so")
 
 # Storage codes understood by the C++ file.
@@ -84,6 +85,13 @@ def _load():
         lib.tbe_oracle_backward_dense.restype = ctypes.c_int
         lib.tbe_oracle_weight_grad.argtypes = [i32, p, p, p, p, i32, p, i32, i64, p, i32, p, i32, p]
         lib.tbe_oracle_weight_grad.restype = ctypes.c_int
+        lib.opt_oracle_double_to_half.argtypes = [ctypes.c_double]
+        lib.opt_oracle_double_to_half.restype = ctypes.c_uint16
+        lib.opt_oracle_double_to_bf16.argtypes = [ctypes.c_double]
+        lib.opt_oracle_double_to_bf16.restype = ctypes.c_uint16
+        lib.opt_oracle_apply.argtypes = [i32, p, p, p, p, i64, p, p, p, i32, ctypes.c_double,
+                                         ctypes.c_double, p]
+        lib.opt_oracle_apply.restype = ctypes.c_int
         lib.fm_oracle_forward.argtypes = [i32, i32, i32, i64, p, p]
         lib.fm_oracle_forward.restype = ctypes.c_int
         lib.fm_oracle_backward.argtypes = [i32, i32, i32, i64, p, p, p]
@@ -285,3 +293,55 @@ def fm_backward(y, grad_fm, num_fields: int) -> np.ndarray:
     if st != OK:
         raise OracleError(st)
     return out
+
+
+# ----------------------------------------------------------------------------- optimizer step
+
+OPTIMIZERS = {"sgd": 0, "adagrad": 1}
+
+
+def double_to_half_bits(x: float) -> int:
+    return int(_load().opt_oracle_double_to_half(float(x)))
+
+
+def double_to_bf16_bits(x: float) -> int:
+    return int(_load().opt_oracle_double_to_bf16(float(x)))
+
+
+def apply_step(tables, batch: int, indices, offsets, grad_out, weights=None, mean: bool = False,
+               kind: str = "sgd", lr: float = 0.01, eps: float = 1e-8, state=None):
+    """One optimizer step on the rows the batch touches (opt_oracle.cpp).
+
+    Returns (new tables as torch CPU tensors of the input dtypes, new state as
+    a list of float32 numpy arrays or None). The inputs are not modified.
+    """
+    import torch
+    arrs = [_table_array(t) for t in tables]
+    work = [a.copy() for a, _ in arrs]
+    T = len(work)
+    rows = np.array([a.shape[0] for a in work], dtype=np.int64)
+    dims = np.array([a.shape[1] for a in work], dtype=np.int32)
+    codes = np.array([c for _, c in arrs], dtype=np.int32)
+    res = backward(rows, dims, batch, indices, offsets, grad_out, weights=weights, mean=mean)
+    uniq = np.ascontiguousarray(res.uniq, dtype=np.int64)
+    goff = np.ascontiguousarray(res.grad_offsets, dtype=np.int64)
+    grads = np.ascontiguousarray(res.grads, dtype=np.float64)
+    st = None
+    st_ptrs = None
+    if kind == "adagrad":
+        st = [np.ascontiguousarray(_np(s_, np.float32)).copy() for s_ in state]
+        st_ptrs = (ctypes.c_void_p * T)(*[a.ctypes.data for a in st])
+    tab_ptrs = (ctypes.c_void_p * T)(*[a.ctypes.data for a in work])
+    rc = _load().opt_oracle_apply(T, ctypes.cast(tab_ptrs, ctypes.c_void_p), _ptr(codes), _ptr(dims),
+                                  _ptr(rows), uniq.shape[0], _ptr(uniq), _ptr(goff), _ptr(grads),
+                                  OPTIMIZERS[kind], float(lr), float(eps),
+                                  None if st_ptrs is None else ctypes.cast(st_ptrs, ctypes.c_void_p))
+    if rc != 0:
+        raise OracleError(BAD_ARG)
+    out = []
+    for a, (_, code) in zip(work, arrs):
+        if code == BF16:
+            out.append(torch.from_numpy(a.view(np.int16)).view(torch.bfloat16))
+        else:
+            out.append(torch.from_numpy(a))
+    return out, st
