@@ -178,6 +178,32 @@ uint64_t cb_tbe_launch_count(const cb_tbe* h);
 /* Short English description of a status code. */
 const char* cb_tbe_status_string(cb_status s);
 
+/* Backward with a row-wise optimizer step fused in place of the gradient
+ * output (not in the paper, which frames its benchmark as training-time but
+ * names no optimizer): the de-duplicated gradient G of every touched row
+ * (exactly what cb_tbe_backward computes) is applied to the table at once and
+ * never written out.
+ *   CB_OPT_SGD:             E[r] <- E[r] - lr * G
+ *   CB_OPT_ROWWISE_ADAGRAD: m[r] <- m[r] + mean_j G[j]^2;
+ *                           E[r] <- E[r] - lr * G / (sqrt(m[r]) + eps)
+ * computed in fp32 and rounded once to the table's storage type (round to
+ * nearest even). THIS CALL WRITES THE TABLES given to cb_tbe_create (and the
+ * state arrays); each touched row is written exactly once, so the result is
+ * deterministic. Untouched rows and their state are left alone.
+ *   batch, indices, num_indices, offsets, per_sample_weights, grad_out: as in
+ *       cb_tbe_backward
+ *   kind   CB_OPT_SGD or CB_OPT_ROWWISE_ADAGRAD
+ *   lr     learning rate (any finite value); eps >= 0 (Adagrad)
+ *   state  Adagrad only: device array of T device pointers, state[t] -> fp32
+ *          [rows_t], the running mean squared gradient of each row (start at 0);
+ *          NULL for SGD
+ * Errors as in cb_tbe_backward; there is no capacity error. */
+typedef enum { CB_OPT_SGD = 0, CB_OPT_ROWWISE_ADAGRAD = 1 } cb_optimizer;
+cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                                const void* offsets, const float* per_sample_weights,
+                                const float* grad_out, cb_optimizer kind, float lr, float eps,
+                                float* const* state, cudaStream_t stream);
+
 /* Gradient with respect to the per-sample weights (not in the paper; the
  * pooled bag above is linear in each weight, so this is its exact derivative):
  *   grad_weights[i] = s_b * sum_j grad_out[b, Doff_t + j] * E_t[indices[i], j]

@@ -267,6 +267,180 @@ cb_status check_common(const cb_tbe* h, int32_t batch, const void* indices, int6
     return CB_OK;
 }
 
+struct ApplyArgs {
+    int kind;
+    float lr;
+    float eps;
+    float* const* state;
+};
+
+// The backward: into the caller's sparse-gradient buffers (g), or, with an
+// optimizer step (a), into the tables themselves.
+cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                        const void* offsets, const float* per_sample_weights, const float* grad_out,
+                        cb_sparse_grad* g, const ApplyArgs* a, cudaStream_t stream) {
+    cb_status st = check_common(h, batch, indices, num_indices, offsets);
+    if (st != CB_OK) return st;
+    const int64_t n = num_indices;
+    if (n >= (int64_t(1) << 30)) return CB_ERR_INVALID_ARG;
+    if (n > 0 && batch > 0 && (!grad_out || (reinterpret_cast<uintptr_t>(grad_out) & 15u)))
+        return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    h->last_stream = stream;
+    h->bwd_timed = false;
+    Problem P = make_problem(h, batch, indices, n, offsets, per_sample_weights);
+    record(h, h->ev_bwd[0], stream);
+    if ((h->flags & CB_VALIDATE) && batch > 0) {
+        launch_validate_offsets(P, h->num_sms, stream);
+        h->launches += 1;
+    }
+    if ((n == 0 || batch == 0) && a) return finish_call(h, stream);  // no row is touched
+    if (n == 0 || batch == 0) {
+        bool ok = cudaMemsetAsync(g->table_offsets, 0, sizeof(int64_t) * (h->T + 1), stream) == cudaSuccess;
+        ok = ok && cudaMemsetAsync(g->num_unique, 0, sizeof(int64_t), stream) == cudaSuccess;
+        ok = ok && cudaMemsetAsync(g->num_floats, 0, sizeof(int64_t), stream) == cudaSuccess;
+        if (g->grads) ok = ok && cudaMemsetAsync(g->grad_offsets, 0, sizeof(int64_t), stream) == cudaSuccess;
+        if (!ok) return CB_ERR_CUDA;
+        return finish_call(h, stream);
+    }
+    st = ensure_workspace(h, batch, n);
+    if (st != CB_OK) return st;
+    Workspace w;
+    layout(h, batch, n, static_cast<char*>(h->ws), &w);
+    Plan Q = make_plan(h, w, true, kBwdChunk);
+    const int64_t bound = n / kBwdChunk + h->T + 1;
+    const bool packed = per_sample_weights != nullptr || h->mode == CB_POOL_MEAN;
+
+    // (1) keys and payloads
+    launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
+    h->launches += 2;
+    if (cudaMemsetAsync(w.hist, 0, w.status_bytes + sizeof(uint32_t) * 4, stream) != cudaSuccess)
+        return CB_ERR_CUDA;
+    KeyGen K;
+    K.keys = w.keys[0];
+    K.vals = w.vals[0];
+    K.packed = packed ? w.packed : nullptr;
+    launch_keygen(P, Q, K, packed, bound, h->num_sms, stream);
+    h->launches += 1;
+    record(h, h->ev_bwd[1], stream);
+
+    // (2) radix sort of each table's range, 8 bits of the row number per pass
+    Plan SQ;
+    SQ.chunk_len = static_cast<int32_t>(kSortTileKeys);
+    SQ.snap_cap = 0;
+    SQ.num_classes = 1;
+    SQ.class_tables = h->d_all_tables;
+    SQ.class_table_start = h->d_all_start;
+    SQ.table_pos = w.sp_table_pos;
+    SQ.ord_chunk_base = w.sp_ord;
+    SQ.class_chunk_base = w.sp_class_base;
+    SQ.chunks = w.sp_tiles;
+    SQ.max_chunks = w.sp_max_tiles;
+    SQ.carry_head = SQ.carry_tail = nullptr;
+    SQ.tail_owner = nullptr;
+    launch_plan(P, SQ, 2, nullptr, nullptr, h->num_sms, true, stream);
+    launch_sort_hist(w.keys[0], w.sp_tiles, w.sp_class_base + 1, w.sp_max_tiles, h->d_tables,
+                     h->passes, w.hist, h->num_sms, stream);
+    launch_sort_bases(w.hist, w.sp_table_pos, h->T, h->passes, w.digit_base, stream);
+    h->launches += 4;
+    int cur = 0;
+    for (int p = 0; p < h->passes; ++p) {
+        SortPass S;
+        S.keys_in = w.keys[cur];
+        S.vals_in = w.vals[cur];
+        S.keys_out = w.keys[cur ^ 1];
+        S.vals_out = w.vals[cur ^ 1];
+        S.tiles = w.sp_tiles;
+        S.num_tiles = w.sp_class_base + 1;
+        S.table_first_tile = w.sp_ord;
+        S.tables = h->d_tables;
+        S.n = n;
+        S.shift = 8 * p;
+        S.digit_base = w.digit_base + 256 * p;
+        S.base_stride = 256 * h->passes;
+        S.status = w.status + static_cast<size_t>(p) * w.sort_tiles * 256;
+        S.tile_counter = w.tile_counters + p;
+        S.never_set = h->d_never_set;
+        S.force_timeout = (h->flags & CB_DEBUG_FORCE_LOOKBACK_TIMEOUT) && p == 0;
+        S.error = h->d_error;
+        S.timeout_ns = kLookbackTimeoutNs;
+        launch_onesweep(S, w.sp_max_tiles, stream);
+        h->launches += 1;
+        cur ^= 1;
+    }
+    record(h, h->ev_bwd[2], stream);
+
+    // (3) runs of equal ids, (4) per-table ranges and capacity check
+    launch_rle(w.keys[cur], n, w.tile_heads, w.tile_base, w.num_unique, w.uniq, w.seg_start, stream);
+    h->launches += 3;
+    BwdOut O;
+    O.seg_start = w.seg_start;
+    O.vals_sorted = w.vals[cur];
+    O.packed = packed ? w.packed : nullptr;
+    O.uniq = w.uniq;
+    O.num_unique_ws = w.num_unique;
+    O.table_first = w.table_first;
+    O.float_base = w.float_base;
+    O.cap_fail = w.cap_fail;
+    O.heavy = w.heavy;
+    O.heavy_count = w.heavy_count;
+    O.max_heavy = w.max_heavy;
+    if (a) {
+        // No caller buffers: the sizes land in the workspace's own words.
+        O.unique_ids = nullptr;
+        O.table_offsets = w.table_first;
+        O.grad_offsets = nullptr;
+        O.grads = nullptr;
+        O.cap_rows = O.cap_floats = INT64_MAX;
+        O.num_unique = w.num_unique;
+        O.num_floats = w.float_base + h->T;
+        O.apply = a->kind;
+        O.lr = a->lr;
+        O.eps = a->eps;
+        O.state = a->state;
+    } else {
+        O.unique_ids = g->unique_ids;
+        O.table_offsets = g->table_offsets;
+        O.grad_offsets = g->grad_offsets;
+        O.grads = g->grads;
+        O.cap_rows = g->cap_rows;
+        O.cap_floats = g->cap_floats;
+        O.num_unique = g->num_unique;
+        O.num_floats = g->num_floats;
+        O.apply = 0;
+        O.lr = O.eps = 0.f;
+        O.state = nullptr;
+    }
+    const bool reduce = a || g->grads;  // a sizing call stops after the run counts
+    launch_bwd_finalize(P, O, stream);
+    h->launches += 1;
+    if (reduce) launch_plan(P, Q, 1, w.seg_start, w.num_unique, h->num_sms, false, stream);
+    if (reduce) h->launches += 1;
+    record(h, h->ev_bwd[3], stream);
+
+    // (5) segmented reduce, (6) fix-up of runs split across chunks
+    if (reduce) {
+        for (size_t c = 0; c < h->bwd_classes.size(); ++c) {
+            if (a)
+                launch_bwd_reduce_apply(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl,
+                                        h->bwd_classes[c].gc, packed, bound, h->num_sms, stream);
+            else
+                launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl,
+                                  h->bwd_classes[c].gc, packed, bound, h->num_sms, stream);
+            h->launches += 1;
+        }
+        launch_bwd_fixup(P, Q, O, bound, h->num_sms, stream);
+        h->launches += 2;
+        if (a) {
+            launch_bwd_apply_split(P, Q, O, bound, h->num_sms, stream);
+            h->launches += 1;
+        }
+    }
+    record(h, h->ev_bwd[4], stream);
+    h->bwd_timed = (h->flags & CB_TIMING) != 0;
+    return finish_call(h, stream);
+}
+
 }  // namespace
 
 extern "C" {
@@ -526,142 +700,29 @@ cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int6
 cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
                           const void* offsets, const float* per_sample_weights,
                           const float* grad_out, cb_sparse_grad* g, cudaStream_t stream) {
-    cb_status st = check_common(h, batch, indices, num_indices, offsets);
-    if (st != CB_OK) return st;
+    if (!h) return CB_ERR_INVALID_ARG;
     if (!g || !g->table_offsets || !g->num_unique || !g->num_floats) return CB_ERR_INVALID_ARG;
     if (g->grads && (!g->unique_ids || !g->grad_offsets || g->cap_rows < 0 || g->cap_floats < 0 ||
                      (reinterpret_cast<uintptr_t>(g->grads) & 15u)))
         return CB_ERR_INVALID_ARG;
-    const int64_t n = num_indices;
-    if (n >= (int64_t(1) << 30)) return CB_ERR_INVALID_ARG;
-    if (n > 0 && batch > 0 && (!grad_out || (reinterpret_cast<uintptr_t>(grad_out) & 15u)))
-        return CB_ERR_INVALID_ARG;
-    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
-    h->last_stream = stream;
-    h->bwd_timed = false;
-    Problem P = make_problem(h, batch, indices, n, offsets, per_sample_weights);
-    record(h, h->ev_bwd[0], stream);
-    if ((h->flags & CB_VALIDATE) && batch > 0) {
-        launch_validate_offsets(P, h->num_sms, stream);
-        h->launches += 1;
-    }
-    if (n == 0 || batch == 0) {
-        bool ok = cudaMemsetAsync(g->table_offsets, 0, sizeof(int64_t) * (h->T + 1), stream) == cudaSuccess;
-        ok = ok && cudaMemsetAsync(g->num_unique, 0, sizeof(int64_t), stream) == cudaSuccess;
-        ok = ok && cudaMemsetAsync(g->num_floats, 0, sizeof(int64_t), stream) == cudaSuccess;
-        if (g->grads) ok = ok && cudaMemsetAsync(g->grad_offsets, 0, sizeof(int64_t), stream) == cudaSuccess;
-        if (!ok) return CB_ERR_CUDA;
-        return finish_call(h, stream);
-    }
-    st = ensure_workspace(h, batch, n);
-    if (st != CB_OK) return st;
-    Workspace w;
-    layout(h, batch, n, static_cast<char*>(h->ws), &w);
-    Plan Q = make_plan(h, w, true, kBwdChunk);
-    const int64_t bound = n / kBwdChunk + h->T + 1;
-    const bool packed = per_sample_weights != nullptr || h->mode == CB_POOL_MEAN;
+    return backward_impl(h, batch, indices, num_indices, offsets, per_sample_weights, grad_out, g, nullptr,
+                         stream);
+}
 
-    // (1) keys and payloads
-    launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
-    h->launches += 2;
-    if (cudaMemsetAsync(w.hist, 0, w.status_bytes + sizeof(uint32_t) * 4, stream) != cudaSuccess)
-        return CB_ERR_CUDA;
-    KeyGen K;
-    K.keys = w.keys[0];
-    K.vals = w.vals[0];
-    K.packed = packed ? w.packed : nullptr;
-    launch_keygen(P, Q, K, packed, bound, h->num_sms, stream);
-    h->launches += 1;
-    record(h, h->ev_bwd[1], stream);
-
-    // (2) radix sort of each table's range, 8 bits of the row number per pass
-    Plan SQ;
-    SQ.chunk_len = static_cast<int32_t>(kSortTileKeys);
-    SQ.snap_cap = 0;
-    SQ.num_classes = 1;
-    SQ.class_tables = h->d_all_tables;
-    SQ.class_table_start = h->d_all_start;
-    SQ.table_pos = w.sp_table_pos;
-    SQ.ord_chunk_base = w.sp_ord;
-    SQ.class_chunk_base = w.sp_class_base;
-    SQ.chunks = w.sp_tiles;
-    SQ.max_chunks = w.sp_max_tiles;
-    SQ.carry_head = SQ.carry_tail = nullptr;
-    SQ.tail_owner = nullptr;
-    launch_plan(P, SQ, 2, nullptr, nullptr, h->num_sms, true, stream);
-    launch_sort_hist(w.keys[0], w.sp_tiles, w.sp_class_base + 1, w.sp_max_tiles, h->d_tables,
-                     h->passes, w.hist, h->num_sms, stream);
-    launch_sort_bases(w.hist, w.sp_table_pos, h->T, h->passes, w.digit_base, stream);
-    h->launches += 4;
-    int cur = 0;
-    for (int p = 0; p < h->passes; ++p) {
-        SortPass S;
-        S.keys_in = w.keys[cur];
-        S.vals_in = w.vals[cur];
-        S.keys_out = w.keys[cur ^ 1];
-        S.vals_out = w.vals[cur ^ 1];
-        S.tiles = w.sp_tiles;
-        S.num_tiles = w.sp_class_base + 1;
-        S.table_first_tile = w.sp_ord;
-        S.tables = h->d_tables;
-        S.n = n;
-        S.shift = 8 * p;
-        S.digit_base = w.digit_base + 256 * p;
-        S.base_stride = 256 * h->passes;
-        S.status = w.status + static_cast<size_t>(p) * w.sort_tiles * 256;
-        S.tile_counter = w.tile_counters + p;
-        S.never_set = h->d_never_set;
-        S.force_timeout = (h->flags & CB_DEBUG_FORCE_LOOKBACK_TIMEOUT) && p == 0;
-        S.error = h->d_error;
-        S.timeout_ns = kLookbackTimeoutNs;
-        launch_onesweep(S, w.sp_max_tiles, stream);
-        h->launches += 1;
-        cur ^= 1;
-    }
-    record(h, h->ev_bwd[2], stream);
-
-    // (3) runs of equal ids, (4) per-table ranges and capacity check
-    launch_rle(w.keys[cur], n, w.tile_heads, w.tile_base, w.num_unique, w.uniq, w.seg_start, stream);
-    h->launches += 3;
-    BwdOut O;
-    O.seg_start = w.seg_start;
-    O.vals_sorted = w.vals[cur];
-    O.packed = packed ? w.packed : nullptr;
-    O.uniq = w.uniq;
-    O.num_unique_ws = w.num_unique;
-    O.table_first = w.table_first;
-    O.float_base = w.float_base;
-    O.cap_fail = w.cap_fail;
-    O.heavy = w.heavy;
-    O.heavy_count = w.heavy_count;
-    O.max_heavy = w.max_heavy;
-    O.unique_ids = g->unique_ids;
-    O.table_offsets = g->table_offsets;
-    O.grad_offsets = g->grad_offsets;
-    O.grads = g->grads;
-    O.cap_rows = g->cap_rows;
-    O.cap_floats = g->cap_floats;
-    O.num_unique = g->num_unique;
-    O.num_floats = g->num_floats;
-    launch_bwd_finalize(P, O, stream);
-    h->launches += 1;
-    if (g->grads) launch_plan(P, Q, 1, w.seg_start, w.num_unique, h->num_sms, false, stream);
-    if (g->grads) h->launches += 1;
-    record(h, h->ev_bwd[3], stream);
-
-    // (5) segmented reduce, (6) fix-up of runs split across chunks
-    if (g->grads) {
-        for (size_t c = 0; c < h->bwd_classes.size(); ++c) {
-            launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl,
-                              h->bwd_classes[c].gc, packed, bound, h->num_sms, stream);
-            h->launches += 1;
-        }
-        launch_bwd_fixup(P, Q, O, bound, h->num_sms, stream);
-        h->launches += 2;
-    }
-    record(h, h->ev_bwd[4], stream);
-    h->bwd_timed = (h->flags & CB_TIMING) != 0;
-    return finish_call(h, stream);
+cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
+                                const void* offsets, const float* per_sample_weights,
+                                const float* grad_out, cb_optimizer kind, float lr, float eps,
+                                float* const* state, cudaStream_t stream) {
+    if (!h) return CB_ERR_INVALID_ARG;
+    if (kind != CB_OPT_SGD && kind != CB_OPT_ROWWISE_ADAGRAD) return CB_ERR_INVALID_ARG;
+    if (!(lr == lr) || !(eps >= 0.f) || (kind == CB_OPT_ROWWISE_ADAGRAD && !state)) return CB_ERR_INVALID_ARG;
+    ApplyArgs a;
+    a.kind = kind == CB_OPT_SGD ? kApplySgd : kApplyAdagrad;
+    a.lr = lr;
+    a.eps = eps;
+    a.state = state;
+    return backward_impl(h, batch, indices, num_indices, offsets, per_sample_weights, grad_out, nullptr, &a,
+                         stream);
 }
 
 cb_status cb_tbe_get_error(cb_tbe* h) {

@@ -10,8 +10,11 @@
 // packed gradient offsets; (5) segmented reduce of the gathered grad_out
 // slices, one warp per chunk of sorted positions; (6) fp64 fix-up of runs that
 // straddle chunks.
+#include <cuda_bf16.h>
+
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
+#include "tbe_reduce.cuh"
 
 namespace cbtbe {
 
@@ -189,123 +192,6 @@ __global__ void __launch_bounds__(1024) bwd_finalize_kernel(Problem P, BwdOut O)
     }
 }
 
-// ---------------------------------------------------------------- (5) reduce
-
-template <int VPL, bool PACKED>
-struct BwdPolicy {
-    static constexpr int kDtype = CB_F32;
-    static constexpr int kElems = 4;
-    static constexpr int kVpl = VPL;
-    static constexpr int kUnroll = CB_REDUCE_ROWS / VPL > 0 ? CB_REDUCE_ROWS / VPL : 1;
-    static constexpr bool kWeighted = PACKED;
-    static constexpr bool kUnrollGroups = CB_REDUCE_UNROLL_GROUPS;
-    static constexpr bool kFastBatch = CB_REDUCE_FAST_BATCH;
-
-    const Problem& P;  // kernel parameters: read in place, not held in registers
-    const Plan& Q;
-    const BwdOut& O;
-    const uint4* base;  // grad_out + Doff_t, one row per bag of this table
-    int64_t float_lo;   // first float of this table in grads
-    uint32_t stride;    // sum of dims / 4
-    int32_t chunk;
-    int32_t bag_lo;
-    int32_t seg_lo;     // first unique index of this table
-    int32_t dim;
-
-    __device__ __forceinline__ int64_t seg_begin(int32_t s) const { return __ldg(O.seg_start + s); }
-    __device__ __forceinline__ int64_t seg_end(int32_t s) const { return __ldg(O.seg_start + s + 1); }
-    struct Raw {
-        uint32_t v;
-    };
-    __device__ __forceinline__ static Raw none() { return {0xffffffffu}; }
-    __device__ __forceinline__ Raw fetch(int64_t q) const { return {__ldg(O.vals_sorted + q)}; }
-    // Sorted item: the bag whose grad_out row it gathers, and w_i * s_b.
-    __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
-        int64_t bag;
-        if (PACKED) {
-            if (x.v >= P.n) {  // only after an aborted sort pass: skip the item
-                a = kInvalid;
-                w = 0.f;
-                return;
-            }
-            const uint2 pk = __ldg(O.packed + x.v);
-            bag = pk.x;
-            w = __uint_as_float(pk.y);
-        } else {
-            bag = x.v;
-            w = 1.f;
-        }
-        const int64_t b = bag - bag_lo;
-        a = (b >= 0 && b < P.B) ? static_cast<uint32_t>(b) : kInvalid;
-    }
-    static constexpr bool kEmptySegments = false;
-    // Row id and float offset of a run that begins in this chunk.
-    __device__ __forceinline__ void seg_meta(int32_t seg) const {
-        O.unique_ids[seg] = __ldg(O.uniq + seg);
-        O.grad_offsets[seg] = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
-    }
-    __device__ __forceinline__ void put_empty(int32_t, int, bool) const {}
-    __device__ __forceinline__ void emit(int32_t seg, int32_t L, bool started, bool ends,
-                                         float (&tot)[VPL][4], int v, bool group0) const {
-        if (started && (threadIdx.x & 31) == 0) seg_meta(seg);
-        put(seg, L, started, ends, tot, v, group0);
-    }
-    __device__ __forceinline__ void put(int32_t seg, int32_t, bool started, bool ends,
-                                        float (&tot)[VPL][4], int v, bool group0) const {
-        const int64_t fo = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
-        if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = seg;
-        if (!group0) return;
-        float* dst;
-        if (started && ends) dst = O.grads + fo;
-        else dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
-#pragma unroll
-        for (int k = 0; k < VPL; ++k) {
-            const int vec = v + 32 * k;
-            if (vec < dim / 4)
-                reinterpret_cast<float4*>(dst)[vec] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
-        }
-    }
-};
-
-template <int VPL, bool PACKED, int GC>
-__global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
-    bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
-                      const __grid_constant__ BwdOut O, const float* grad_out, int cls) {
-    if (*O.cap_fail) return;
-    const int lane = threadIdx.x & 31;
-    const int64_t cb = Q.class_chunk_base[cls];
-    const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
-    for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
-        const Chunk ch = Q.chunks[j];
-        const int t = ch.table;
-        const TableDev& td = P.tables[t];
-        BwdPolicy<VPL, PACKED> pol{P, Q, O};
-        pol.base = reinterpret_cast<const uint4*>(grad_out + td.doff);
-        pol.float_lo = O.float_base[t];
-        pol.stride = static_cast<uint32_t>(P.sum_d / 4);
-        pol.chunk = static_cast<int32_t>(j);
-        pol.bag_lo = t * P.B;
-        pol.seg_lo = static_cast<int32_t>(O.table_first[t]);
-        pol.dim = td.dim;
-        ChunkCtx c;
-        c.k0 = ch.k0;
-        c.len = static_cast<int32_t>(ch.len & 0x7fffffffu);
-        c.first = static_cast<int32_t>(max64(ch.first, O.table_first[t]));
-        c.seg_hi = static_cast<int32_t>(O.table_first[t + 1]);
-        c.lanes = td.grad_lanes;
-        c.groups = td.grad_groups;
-        c.row_vecs = td.grad_vecs;
-        c.last = false;
-        if (lane == 0) Q.tail_owner[j] = -1;
-        if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
-            __shared__ EndSlot slots[kWarpThreads / 32][32];
-            walk_rows<BwdPolicy<VPL, PACKED>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
-        } else {
-            walk_chunk<BwdPolicy<VPL, PACKED>, GC>(pol, c, P.zero_row, lane);
-        }
-    }
-}
-
 // ---------------------------------------------------------------- (6) fix-up
 
 // Runs split over chunks (hot rows longer than the snap cap): each warp scans
@@ -345,7 +231,9 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(const __grid_co
             }
             const int t = Q.chunks[j].table;
             const TableDev& td = P.tables[t];
-            float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
+            // A fused step takes the combined row from the chunk's tail slot.
+            float* dst = O.apply ? Q.carry_tail + j * P.dmax
+                                 : O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
             combine_pieces(Q, j, m, td.dim, P.dmax, lane,
                            [&](int x0, double (&acc)[4]) { store_grad4(dst, x0, acc); });
         }
@@ -383,7 +271,8 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_heavy_kernel(const __grid_co
         }
         __syncthreads();
         if (w == 0) {
-            float* dst = O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
+            float* dst = O.apply ? Q.carry_tail + j * P.dmax
+                                 : O.grads + O.float_base[t] + (seg - O.table_first[t]) * td.dim;
             const float* tail = Q.carry_tail + j * P.dmax;
             for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
                 const float4 a = *reinterpret_cast<const float4*>(tail + x0);
@@ -397,21 +286,37 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_heavy_kernel(const __grid_co
     }
 }
 
+// Fused step for the runs the fix-up combined: their full gradient row waits in
+// the tail slot of the chunk where the run begins. One warp per such run.
+__global__ void __launch_bounds__(kWarpThreads) bwd_apply_split_kernel(const __grid_constant__ Problem P,
+                                                                       const __grid_constant__ Plan Q,
+                                                                       const __grid_constant__ BwdOut O) {
+    if (*O.cap_fail) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
+    for (int64_t base = warp_id_global() * 32; base < total; base += warps_in_grid() * 32) {
+        const int64_t mine = base + lane < total ? Q.tail_owner[base + lane] : -1;
+        for (uint32_t mask = __ballot_sync(kFull, mine >= 0); mask; mask &= mask - 1) {
+            const int b = __ffs(mask) - 1;
+            const int64_t j = base + b;
+            const int64_t seg = __shfl_sync(kFull, mine, b);
+            const int t = Q.chunks[j].table;
+            const TableDev& td = P.tables[t];
+            const int64_t row = static_cast<int64_t>(O.uniq[seg]) - td.row_base;
+            const float* g = Q.carry_tail + j * P.dmax;
+            float sq = 0.f;
+            for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
+                const float4 v = *reinterpret_cast<const float4*>(g + x0);
+                sq += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+            }
+            const float scale = step_scale(O, t, row, td.dim, sq);
+            for (int x0 = lane * 4; x0 < td.dim; x0 += 128)
+                step_cols(td, row, x0, *reinterpret_cast<const float4*>(g + x0), scale);
+        }
+    }
+}
+
 // ---------------------------------------------------------------- launchers
-
-template <class KernelT>
-static int occupancy_grid(KernelT kernel, int threads, int num_sms) {
-    int per_sm = 1;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0) != cudaSuccess ||
-        per_sm < 1)
-        per_sm = 1;
-    return per_sm * num_sms;
-}
-
-static int warp_grid(int64_t chunk_bound, int cap) {
-    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
-    return static_cast<int>(max64(1, min64(need, cap)));
-}
 
 void launch_keygen(const Problem& P, const Plan& Q, const KeyGen& K, bool packed, int64_t chunk_bound,
                    int num_sms, cudaStream_t s) {
@@ -439,26 +344,10 @@ void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s) {
     bwd_finalize_kernel<<<1, 1024, 0, s>>>(P, O);
 }
 
-template <int VPL, bool PACKED, int GC>
-static void launch_reduce_one(const Problem& P, const Plan& Q, const BwdOut& O, const float* go,
-                              int cls, int64_t chunk_bound, int num_sms, cudaStream_t s) {
-    static int cap = occupancy_grid(bwd_reduce_kernel<VPL, PACKED, GC>, kWarpThreads, num_sms);
-    bwd_reduce_kernel<VPL, PACKED, GC><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, O, go, cls);
-}
-
 void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
                        int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
                        cudaStream_t s) {
-#define CB_CASE(V, G, PK)                                                                \
-    if (vpl == V && gc == G && packed == PK) {                                            \
-        launch_reduce_one<V, PK, G>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s);    \
-        return;                                                                          \
-    }
-    CB_CASE(1, 1, false) CB_CASE(1, 2, false) CB_CASE(1, 4, false) CB_CASE(1, 8, false)
-    CB_CASE(1, 0, false) CB_CASE(2, 1, false) CB_CASE(4, 1, false)
-    CB_CASE(1, 1, true) CB_CASE(1, 2, true) CB_CASE(1, 4, true) CB_CASE(1, 8, true)
-    CB_CASE(1, 0, true) CB_CASE(2, 1, true) CB_CASE(4, 1, true)
-#undef CB_CASE
+    launch_bwd_reduce_t<false>(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
 }
 
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
@@ -469,6 +358,13 @@ void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t 
     bwd_fixup_kernel<<<grid, kWarpThreads, 0, s>>>(P, Q, O);
     const int hgrid = static_cast<int>(max64(1, min64(O.max_heavy, static_cast<int64_t>(num_sms) * 4)));
     bwd_heavy_kernel<<<hgrid, kWarpThreads, 0, s>>>(P, Q, O);
+}
+
+void launch_bwd_apply_split(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
+                            int num_sms, cudaStream_t s) {
+    const int64_t need = (chunk_bound + kWarpThreads - 1) / kWarpThreads;  // 32 chunks per warp
+    const int grid = static_cast<int>(max64(1, min64(need, static_cast<int64_t>(num_sms) * 8)));
+    bwd_apply_split_kernel<<<grid, kWarpThreads, 0, s>>>(P, Q, O);
 }
 
 }  // namespace cbtbe

@@ -60,7 +60,15 @@ struct BwdOut {
     int64_t cap_floats;
     int64_t* num_unique;
     int64_t* num_floats;
+    // Optimizer step fused in place of the gradient output (apply != 0): no
+    // gradient buffers; every touched table row is updated where its sum ends.
+    int apply;             // 0: write gradients, kApplySgd, kApplyAdagrad
+    float lr;
+    float eps;
+    float* const* state;   // device [T] -> fp32 [rows_t] (row-wise Adagrad)
 };
+constexpr int kApplySgd = 1;
+constexpr int kApplyAdagrad = 2;
 
 void launch_validate_offsets(const Problem& P, int num_sms, cudaStream_t s);
 void launch_plan(const Problem& P, const Plan& Q, int mode, const uint32_t* seg_start,
@@ -97,7 +105,12 @@ inline int compile_time_groups(int vpl, int lanes, int groups) {
 }
 void launch_weight_grad(const Problem& P, const Plan& Q, const float* grad_out, float* grad_w, int cls,
                         int dtype, int gc, int64_t chunk_bound, int num_sms, cudaStream_t s);
+void launch_bwd_reduce_apply(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
+                             int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
+                             cudaStream_t s);
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
+void launch_bwd_apply_split(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
+                            int num_sms, cudaStream_t s);
 
 }  // namespace cbtbe

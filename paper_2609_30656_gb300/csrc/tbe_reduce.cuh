@@ -1,0 +1,263 @@
+// tbe_reduce.cuh -- the backward segmented reduce (runs of equal sorted row
+// ids; per run the coefficient-weighted sum of the gathered grad_out slices,
+// the de-duplicated adjoint of the pooled bag of Sec. IV.A.2), and the
+// optimizer step that can be fused where a run's sum ends. Included by
+// tbe_backward.cu (gradient output) and tbe_backward_apply.cu (fused step).
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include "tbe_internal.cuh"
+#include "tbe_launch.h"
+
+namespace cbtbe {
+
+template <class KernelT>
+inline int occupancy_grid(KernelT kernel, int threads, int num_sms) {
+    int per_sm = 1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0) != cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    return per_sm * num_sms;
+}
+
+inline int warp_grid(int64_t chunk_bound, int cap) {
+    const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
+    return static_cast<int>(max64(1, min64(need, cap)));
+}
+
+// ---------------------------------------------------------------- optimizer step
+
+// new = E - scale * g for four consecutive columns of a stored row, rounded
+// once from fp32 to the storage type (round to nearest even).
+__device__ __forceinline__ void step_cols(const TableDev& td, int64_t row, int col, float4 g, float scale) {
+    const int64_t k = row * td.dim + col;
+    if (td.dtype == CB_F32) {
+        float4* p = reinterpret_cast<float4*>(const_cast<void*>(td.data)) + k / 4;
+        float4 x = *p;
+        x.x = fmaf(-scale, g.x, x.x);
+        x.y = fmaf(-scale, g.y, x.y);
+        x.z = fmaf(-scale, g.z, x.z);
+        x.w = fmaf(-scale, g.w, x.w);
+        *p = x;
+    } else if (td.dtype == CB_F16) {
+        uint2* p = reinterpret_cast<uint2*>(const_cast<void*>(td.data)) + k / 4;
+        uint2 x = *p;
+        __half2 a, b;
+        memcpy(&a, &x.x, 4);
+        memcpy(&b, &x.y, 4);
+        const float2 fa = __half22float2(a), fb = __half22float2(b);
+        a = __floats2half2_rn(fmaf(-scale, g.x, fa.x), fmaf(-scale, g.y, fa.y));
+        b = __floats2half2_rn(fmaf(-scale, g.z, fb.x), fmaf(-scale, g.w, fb.y));
+        memcpy(&x.x, &a, 4);
+        memcpy(&x.y, &b, 4);
+        *p = x;
+    } else {
+        uint2* p = reinterpret_cast<uint2*>(const_cast<void*>(td.data)) + k / 4;
+        uint2 x = *p;
+        const float f0 = __uint_as_float(x.x << 16), f1 = __uint_as_float(x.x & 0xffff0000u);
+        const float f2 = __uint_as_float(x.y << 16), f3 = __uint_as_float(x.y & 0xffff0000u);
+        const __nv_bfloat162 a = __floats2bfloat162_rn(fmaf(-scale, g.x, f0), fmaf(-scale, g.y, f1));
+        const __nv_bfloat162 b = __floats2bfloat162_rn(fmaf(-scale, g.z, f2), fmaf(-scale, g.w, f3));
+        memcpy(&x.x, &a, 4);
+        memcpy(&x.y, &b, 4);
+        *p = x;
+    }
+}
+
+// The step's scale for one row: lr (SGD), or lr / (sqrt(m) + eps) after
+// m += mean of the squared gradient (row-wise Adagrad). `sq` is this lane's
+// share of sum g^2; the whole warp calls this, lane 0 owns the state word.
+__device__ __forceinline__ float step_scale(const BwdOut& O, int t, int64_t row, int dim, float sq) {
+    if (O.apply != kApplyAdagrad) return O.lr;
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) sq += __shfl_xor_sync(kFull, sq, off);
+    float m = 0.f;
+    if ((threadIdx.x & 31) == 0) {
+        float* st = O.state[t] + row;
+        m = *st + sq / static_cast<float>(dim);
+        *st = m;
+    }
+    m = __shfl_sync(kFull, m, 0);
+    return O.lr / (sqrtf(m) + O.eps);
+}
+
+// The fused step on one complete run's row, as the walker holds it: lane v of
+// each row group owns vectors v + 32k; every group holds the same totals and
+// group 0 writes.
+template <int VPL>
+struct GradRow {
+    float4 v[VPL];
+};
+
+template <int VPL>
+__device__ __forceinline__ void apply_row(const Problem& P, const BwdOut& O, int t, int32_t seg,
+                                          const GradRow<VPL>& g, int v, bool group0) {
+    const TableDev& td = P.tables[t];
+    const int64_t row = static_cast<int64_t>(__ldg(O.uniq + seg)) - td.row_base;
+    const int nv = td.dim / 4;
+    float sq = 0.f;
+#pragma unroll
+    for (int k = 0; k < VPL; ++k)
+        if (group0 && v + 32 * k < nv)
+            sq += g.v[k].x * g.v[k].x + g.v[k].y * g.v[k].y + g.v[k].z * g.v[k].z + g.v[k].w * g.v[k].w;
+    const float scale = step_scale(O, t, row, td.dim, sq);
+    if (!group0) return;
+#pragma unroll
+    for (int k = 0; k < VPL; ++k)
+        if (v + 32 * k < nv) step_cols(td, row, 4 * (v + 32 * k), g.v[k], scale);
+}
+
+// ---------------------------------------------------------------- (5) reduce
+
+// APPLY: the optimizer step is fused where a run's sum ends (compiled as its
+// own kernels, so the gradient-writing reduce carries none of its code).
+template <int VPL, bool PACKED, bool APPLY>
+struct BwdPolicy {
+    static constexpr int kDtype = CB_F32;
+    static constexpr int kElems = 4;
+    static constexpr int kVpl = VPL;
+    static constexpr int kUnroll = CB_REDUCE_ROWS / VPL > 0 ? CB_REDUCE_ROWS / VPL : 1;
+    static constexpr bool kWeighted = PACKED;
+    static constexpr bool kUnrollGroups = CB_REDUCE_UNROLL_GROUPS;
+    static constexpr bool kFastBatch = CB_REDUCE_FAST_BATCH;
+
+    const Problem& P;  // kernel parameters: read in place, not held in registers
+    const Plan& Q;
+    const BwdOut& O;
+    const uint4* base;  // grad_out + Doff_t, one row per bag of this table
+    int64_t float_lo;   // first float of this table in grads
+    uint32_t stride;    // sum of dims / 4
+    int32_t chunk;
+    int32_t bag_lo;
+    int32_t seg_lo;     // first unique index of this table
+    int32_t dim;
+    int32_t table;
+
+    __device__ __forceinline__ int64_t seg_begin(int32_t s) const { return __ldg(O.seg_start + s); }
+    __device__ __forceinline__ int64_t seg_end(int32_t s) const { return __ldg(O.seg_start + s + 1); }
+    struct Raw {
+        uint32_t v;
+    };
+    __device__ __forceinline__ static Raw none() { return {0xffffffffu}; }
+    __device__ __forceinline__ Raw fetch(int64_t q) const { return {__ldg(O.vals_sorted + q)}; }
+    // Sorted item: the bag whose grad_out row it gathers, and w_i * s_b.
+    __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
+        int64_t bag;
+        if (PACKED) {
+            if (x.v >= P.n) {  // only after an aborted sort pass: skip the item
+                a = kInvalid;
+                w = 0.f;
+                return;
+            }
+            const uint2 pk = __ldg(O.packed + x.v);
+            bag = pk.x;
+            w = __uint_as_float(pk.y);
+        } else {
+            bag = x.v;
+            w = 1.f;
+        }
+        const int64_t b = bag - bag_lo;
+        a = (b >= 0 && b < P.B) ? static_cast<uint32_t>(b) : kInvalid;
+    }
+    static constexpr bool kEmptySegments = false;
+    // Row id and float offset of a run that begins in this chunk.
+    __device__ __forceinline__ void seg_meta(int32_t seg) const {
+        if (APPLY) return;  // a fused step writes no gradient buffers
+        O.unique_ids[seg] = __ldg(O.uniq + seg);
+        O.grad_offsets[seg] = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
+    }
+    __device__ __forceinline__ void put_empty(int32_t, int, bool) const {}
+    __device__ __forceinline__ void emit(int32_t seg, int32_t L, bool started, bool ends,
+                                         float (&tot)[VPL][4], int v, bool group0) const {
+        if (started && (threadIdx.x & 31) == 0) seg_meta(seg);
+        put(seg, L, started, ends, tot, v, group0);
+    }
+    __device__ __forceinline__ void put(int32_t seg, int32_t, bool started, bool ends,
+                                        float (&tot)[VPL][4], int v, bool group0) const {
+        const int64_t fo = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
+        if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = seg;
+        if (APPLY && started && ends) {
+            GradRow<VPL> r;
+#pragma unroll
+            for (int k = 0; k < VPL; ++k) r.v[k] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
+            apply_row<VPL>(P, O, table, seg, r, v, group0);
+            return;
+        }
+        if (!group0) return;
+        float* dst;
+        if (started && ends) dst = O.grads + fo;
+        else dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
+#pragma unroll
+        for (int k = 0; k < VPL; ++k) {
+            const int vec = v + 32 * k;
+            if (vec < dim / 4)
+                reinterpret_cast<float4*>(dst)[vec] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
+        }
+    }
+};
+
+template <int VPL, bool PACKED, int GC, bool APPLY>
+__global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
+    bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
+                      const __grid_constant__ BwdOut O, const float* grad_out, int cls) {
+    if (*O.cap_fail) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t cb = Q.class_chunk_base[cls];
+    const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
+    for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
+        const Chunk ch = Q.chunks[j];
+        const int t = ch.table;
+        const TableDev& td = P.tables[t];
+        BwdPolicy<VPL, PACKED, APPLY> pol{P, Q, O};
+        pol.base = reinterpret_cast<const uint4*>(grad_out + td.doff);
+        pol.float_lo = O.float_base[t];
+        pol.stride = static_cast<uint32_t>(P.sum_d / 4);
+        pol.chunk = static_cast<int32_t>(j);
+        pol.bag_lo = t * P.B;
+        pol.seg_lo = static_cast<int32_t>(O.table_first[t]);
+        pol.dim = td.dim;
+        pol.table = t;
+        ChunkCtx c;
+        c.k0 = ch.k0;
+        c.len = static_cast<int32_t>(ch.len & 0x7fffffffu);
+        c.first = static_cast<int32_t>(max64(ch.first, O.table_first[t]));
+        c.seg_hi = static_cast<int32_t>(O.table_first[t + 1]);
+        c.lanes = td.grad_lanes;
+        c.groups = td.grad_groups;
+        c.row_vecs = td.grad_vecs;
+        c.last = false;
+        if (lane == 0) Q.tail_owner[j] = -1;
+        if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
+            __shared__ EndSlot slots[kWarpThreads / 32][32];
+            walk_rows<BwdPolicy<VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+        } else {
+            walk_chunk<BwdPolicy<VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane);
+        }
+    }
+}
+
+template <int VPL, bool PACKED, int GC, bool APPLY>
+static void launch_reduce_one(const Problem& P, const Plan& Q, const BwdOut& O, const float* go,
+                              int cls, int64_t chunk_bound, int num_sms, cudaStream_t s) {
+    static int cap = occupancy_grid(bwd_reduce_kernel<VPL, PACKED, GC, APPLY>, kWarpThreads, num_sms);
+    bwd_reduce_kernel<VPL, PACKED, GC, APPLY><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, O, go, cls);
+}
+
+template <bool APPLY>
+void launch_bwd_reduce_t(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
+                         int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
+                         cudaStream_t s) {
+#define CB_CASE(V, G, PK)                                                                \
+    if (vpl == V && gc == G && packed == PK) {                                            \
+        launch_reduce_one<V, PK, G, APPLY>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s);    \
+        return;                                                                          \
+    }
+    CB_CASE(1, 1, false) CB_CASE(1, 2, false) CB_CASE(1, 4, false) CB_CASE(1, 8, false)
+    CB_CASE(1, 0, false) CB_CASE(2, 1, false) CB_CASE(4, 1, false)
+    CB_CASE(1, 1, true) CB_CASE(1, 2, true) CB_CASE(1, 4, true) CB_CASE(1, 8, true)
+    CB_CASE(1, 0, true) CB_CASE(2, 1, true) CB_CASE(4, 1, true)
+#undef CB_CASE
+}
+
+}  // namespace cbtbe

@@ -29,7 +29,8 @@ _IDX = {torch.int32: 0, torch.int64: 1}
 EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
-           "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad")
+           "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad",
+           "cb_tbe_backward_apply")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -79,11 +80,13 @@ def load_library() -> ctypes.CDLL:
     lib.cb_tbe_destroy.argtypes = [p]
     lib.cb_tbe_destroy.restype = None
     lib.cb_tbe_weight_grad.argtypes = [p, i32, p, i64, p, p, p, p]
+    lib.cb_tbe_backward_apply.argtypes = [p, i32, p, i64, p, p, p, ctypes.c_int, ctypes.c_float,
+                                          ctypes.c_float, p, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
                  "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward",
-                 "cb_tbe_weight_grad"):
+                 "cb_tbe_weight_grad", "cb_tbe_backward_apply"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -253,6 +256,38 @@ class TBE:
         U, F = probe.num_unique, probe.num_floats
         g = self.alloc_grad(U, F)
         return self.backward_into(g, indices, offsets, grad_out, per_sample_weights)
+
+    def backward_apply(self, indices, offsets, grad_out, per_sample_weights=None,
+                       optimizer: str = "sgd", lr: float = 0.01, eps: float = 1e-8,
+                       state: list[torch.Tensor] | None = None) -> None:
+        """Backward with the optimizer step fused (cb_tbe_backward_apply): updates the
+        tables this handle was created with (and, for "adagrad", the fp32 [rows_t]
+        state tensors) in place."""
+        kinds = {"sgd": 0, "adagrad": 1}
+        if optimizer not in kinds:
+            raise ValueError(f"unknown optimizer {optimizer!r}")
+        T = len(self.dims)
+        batch = (offsets.numel() - 1) // T
+        ind = self._dev(indices, self.index_dtype)
+        off = self._dev(offsets, self.index_dtype)
+        w = self._dev(per_sample_weights, torch.float32)
+        go = self._dev(grad_out, torch.float32)
+        ptrs = None
+        if optimizer == "adagrad":
+            if state is None or len(state) != T:
+                raise ValueError("adagrad needs one fp32 state tensor per table")
+            for s_, r in zip(state, self.rows):
+                if (s_.device != self.device or s_.dtype != torch.float32 or s_.numel() != r
+                        or not s_.is_contiguous()):
+                    raise ValueError("state[t] must be a contiguous fp32 [rows_t] tensor on the device")
+            ptrs = torch.tensor([s_.data_ptr() for s_ in state], dtype=torch.int64,
+                                device=self.device)
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_backward_apply(self._h, batch, _ptr(ind), ind.numel(), _ptr(off),
+                                                   _ptr(w), _ptr(go), kinds[optimizer], lr, eps,
+                                                   _ptr(ptrs), self._stream()),
+                   "cb_tbe_backward_apply")
+        self._keep = ptrs  # the pointer array must outlive the enqueued work
 
     def weight_grad(self, indices, offsets, grad_out,
                     out: torch.Tensor | None = None) -> torch.Tensor:

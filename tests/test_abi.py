@@ -73,6 +73,10 @@ def test_host_side_argument_errors_return_before_any_gpu_work(lib):
     assert lib.cb_fm_backward(None, None, 0, 0, 8, 0, None, None) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_fm_backward(None, None, 4, 2, 8, 12, None, None) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_fm_forward(None, 0, 2, 8, 16, None, None) == tbe.CB_OK  # nothing to do
+    # weight gradient and the fused optimizer step on a null handle
+    assert lib.cb_tbe_weight_grad(None, 1, None, 0, None, None, None, None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_backward_apply(None, 1, None, 0, None, None, None, 0, 0.1, 0.0, None,
+                                     None) == tbe.CB_ERR_INVALID_ARG
 
 
 def test_product_path_fails_loudly_without_the_library(monkeypatch, tmp_path):
