@@ -396,6 +396,9 @@ def run_ours(args):
         if len(set(w.dims)) == 1:
             nxt["fm"] = run_fm(w, out, flush, dev, peak)
         nxt["weight_grad"] = run_weight_grad(m, batches[0], grads_out[0], counts[0], flush, peak)
+        # last: it writes the tables
+        nxt["backward_apply"] = run_backward_apply(m, w, batches[0], grads_out[0], counts[0],
+                                                   uniq_tables[0], flush, peak, dev)
         line["next_rows"] = nxt
     # End to end through the public API from pinned host memory.
     if not args.no_e2e:
@@ -509,6 +512,38 @@ def run_weight_grad(m, b, go, c, flush, peak):
             "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes,
             "note": "algorithmic bytes count each lookup's row and grad_out slice; "
                     "repeated rows and a table's grad_out slice are largely served by L2"}
+
+
+def run_backward_apply(m, w, b, go, c, uniq, flush, peak, dev):
+    """Backward with SGD / row-wise Adagrad fused (cb_tbe_backward_apply) on one batch.
+    It updates the bench's synthetic tables in place, so it runs after every other
+    measurement."""
+    state = [torch.zeros(r, dtype=torch.float32, device=dev) for r in w.rows]
+    res = {}
+    for kind in ("sgd", "adagrad"):
+        def call():
+            m.backward_apply(b.indices, b.offsets, go, b.weights, optimizer=kind, lr=1e-3,
+                             eps=1e-8, state=state if kind == "adagrad" else None)
+        for _ in range(2):
+            call()
+        torch.cuda.synchronize()
+        reps = 5
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for a, e in ev:
+            flush.zero_()
+            a.record()
+            call()
+            e.record()
+        torch.cuda.synchronize()
+        if m.get_error() != 0:
+            raise RuntimeError("device-side error in the fused optimizer step")
+        ms = statistics.mean(a.elapsed_time(e) for a, e in ev)
+        nbytes = metrics.apply_step_bytes(c, uniq, kind == "adagrad")
+        res[kind] = {"ms": round(ms, 4), "alg_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
+                     "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes}
+    del state
+    return res
 
 
 def run_fm_only(args):

@@ -15,6 +15,8 @@ result table (Sec. IV.A.1) divided by the achieved time gives the same
             + idx_bytes + 4 (the gradient)    per bag: idx_bytes
   FM cross term    per pooled value: 4 read (+ 4 written by the backward);
             per sample: 4 (fm written, or grad_fm read)
+  fused optimizer step   the backward's reads; per touched row D_t * e_S read
+            and written (+ 8 for the Adagrad state word) instead of the gradient
 """
 
 from __future__ import annotations
@@ -91,6 +93,17 @@ def weight_grad_bytes(c: BatchCounts) -> int:
     rows = sum(L * d * c.elem_bytes for L, d in zip(c.lookups_per_table, c.dims))
     slices = sum(L * d * 4 for L, d in zip(c.lookups_per_table, c.dims))
     return rows + slices + c.n * (c.idx_bytes + 4) + (c.num_tables * c.batch + 1) * c.idx_bytes
+
+
+def apply_step_bytes(c: BatchCounts, unique_per_table, adagrad: bool) -> int:
+    """Algorithmic bytes of the backward with the optimizer step fused: the
+    backward's reads, and each touched row read and written in its storage
+    type (plus its fp32 state word for row-wise Adagrad) instead of the
+    gradient rows and ids."""
+    b = backward_bytes(c, unique_per_table)
+    rows = sum(int(u) * d * c.elem_bytes for u, d in zip(unique_per_table, c.dims))
+    U = int(sum(int(u) for u in unique_per_table))
+    return (b["total"] - b["grads"] - b["unique_ids"] + 2 * rows + (8 * U if adagrad else 0))
 
 
 def sort_bytes(n: int, passes: int) -> int:

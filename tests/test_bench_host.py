@@ -36,6 +36,15 @@ def test_weight_grad_bytes_by_hand():
     assert metrics.weight_grad_bytes(c) == rows + slices + 7 * (8 + 4) + 7 * 8
 
 
+def test_apply_step_bytes_by_hand():
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts((4, 8), 2, 3, off, weighted=False)
+    b = metrics.backward_bytes(c, [3, 1])
+    rows = 3 * 4 * 2 + 1 * 8 * 2
+    assert metrics.apply_step_bytes(c, [3, 1], False) == b["total"] - b["grads"] - b["unique_ids"] + 2 * rows
+    assert metrics.apply_step_bytes(c, [3, 1], True) == metrics.apply_step_bytes(c, [3, 1], False) + 4 * 8
+
+
 def test_fm_bytes_by_hand():
     # 3 samples x 2 fields x dim 4: 24 floats of pooled rows
     assert metrics.fm_bytes(3, 2, 4, backward=False) == 24 * 4 + 3 * 4
