@@ -400,6 +400,9 @@ def run_ours(args):
         nxt["backward_apply"] = run_backward_apply(m, w, batches[0], grads_out[0], counts[0],
                                                    uniq_tables[0], flush, peak, dev)
         line["next_rows"] = nxt
+    # Component report (Component Benchmark's result table) of this run.
+    if args.report and rank == 0:
+        write_report(args.report, w, line, comp_ms, comp_bytes, counts, uniq_tables, peak)
     # End to end through the public API from pinned host memory.
     if not args.no_e2e:
         line["e2e"] = run_e2e(args, m, w, batches, grads_out, g, out, dev, world)
@@ -544,6 +547,46 @@ def run_backward_apply(m, w, b, go, c, uniq, flush, peak, dev):
                      "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes}
     del state
     return res
+
+
+def write_report(path, w, line, comp_ms, comp_bytes, counts, uniq_tables, peak):
+    """Hierarchical component report (JSON and Markdown) of the measured step."""
+    from paper_2609_30656_gb300 import report
+    steps = len(counts)
+    flops = {}
+    for c, u in zip(counts, uniq_tables):
+        for k, v in metrics.component_flops(c, u, w.mean).items():
+            flops[k] = flops.get(k, 0.0) + v / steps
+    per_bytes = {k: v / line["steps"] for k, v in comp_bytes.items()}
+    extra = {}
+    nxt = line.get("next_rows", {})
+    if "fm" in nxt:
+        B, T, D = w.batch, w.num_tables, w.dims[0]
+        extra["fm.forward"] = (nxt["fm"]["forward"]["ms"], nxt["fm"]["forward"]["bytes"], 3.0 * B * T * D)
+        extra["fm.backward"] = (nxt["fm"]["backward"]["ms"], nxt["fm"]["backward"]["bytes"], 2.0 * B * T * D)
+    if "weight_grad" in nxt:
+        g = nxt["weight_grad"]
+        extra["weight_grad"] = (g["ms"], g["bytes"], 2.0 * sum(L * d for L, d in zip(counts[0].lookups_per_table, w.dims)))
+    for kind in ("sgd", "adagrad"):
+        if kind in nxt.get("backward_apply", {}):
+            a = nxt["backward_apply"][kind]
+            extra[f"backward_apply.{kind}"] = (a["ms"], a["bytes"], flops.get("bwd.reduce", 0.0))
+    table_mb = sum(r * d * w.elem_bytes for r, d in zip(w.rows, w.dims)) / 1e6
+    root = report.step_tree(comp_ms, per_bytes, flops, table_mb=table_mb, workspace_mb=0.0,
+                            extra=extra or None)
+    root.latency_ms = line["ms_per_step"]
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            tflops = float(json.load(f)["bf16_tflops"])
+    except Exception:
+        tflops = 1900.0
+    meta = {"workload": line["config"]["workload"],
+            "note": "bytes and FLOPs are algorithmic; BW util against the measured HBM copy "
+                    "bandwidth, MFU against the measured dense bf16 tensor peak"}
+    with open(path + ".json", "w") as f:
+        f.write(report.to_json(root, peak, tflops, **meta))
+    with open(path + ".md", "w") as f:
+        f.write(report.to_markdown(root, peak, tflops, title=f"Component report: {w.name}"))
 
 
 def run_fm_only(args):
@@ -701,6 +744,8 @@ def main(argv=None):
                     help="skip the forward on uniform indices over the same tables")
     ap.add_argument("--no-next", action="store_true",
                     help="skip the next-row measurements (FM cross term)")
+    ap.add_argument("--report", default=None,
+                    help="write a hierarchical component report to REPORT.json and REPORT.md")
     ap.add_argument("--fm-only", action="store_true",
                     help="time only the FM cross term and its gradient on a synthetic pooled "
                          "output of the workload's shape (no tables are allocated)")

@@ -141,3 +141,16 @@ def fm_bytes(batch: int, num_fields: int, dim: int, backward: bool) -> int:
     plus fm [B] written (forward), or grad_fm [B] read and grad_y written (backward)."""
     y = 4 * batch * num_fields * dim
     return y + 4 * batch + (y if backward else 0)
+
+
+def component_flops(c: BatchCounts, unique_per_table, mean: bool) -> dict[str, int]:
+    """Algorithmic floating-point operations of each timed component: one add (or
+    a multiply-add, 2, with weights or mean coefficients) per gathered value, a
+    division per pooled value for mean pooling; the integer stages do none."""
+    per_value = 2 if (c.weighted or mean) else 1
+    gathered = sum(L * d for L, d in zip(c.lookups_per_table, c.dims))
+    return {
+        "fwd.prep": 0, "fwd.fixup": 0, "bwd.keygen": 0, "bwd.sort": 0, "bwd.rle": 0,
+        "fwd.gather": per_value * gathered + (c.batch * c.sum_dims if mean else 0),
+        "bwd.reduce": per_value * gathered,
+    }

@@ -117,3 +117,28 @@ def test_aggregate_takes_max_time_and_summed_work_over_two_gloo_ranks():
 
 def test_aggregate_is_identity_on_one_rank():
     assert bench.aggregate(1.5, 2.0, 3.0, 1) == (1.5, 2.0, 3.0)
+
+
+def test_report_written_from_measured_components(tmp_path):
+    import json
+    w = wl.scaled(wl.get_workload("cfg5"), num_tables=2, batch=3, rows=10)
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, off, weighted=False)
+    comp_ms = {"fwd.prep": 0.01, "fwd.gather": 1.0, "fwd.fixup": 0.01, "bwd.keygen": 0.2,
+               "bwd.sort": 0.5, "bwd.rle": 0.1, "bwd.reduce": 2.0}
+    comp_bytes = {"fwd.gather": 3 * 6e9, "bwd.reduce": 3 * 8e9}  # over the 3 timed steps
+    line = {"steps": 3, "ms_per_step": 4.0, "config": {"workload": "tiny"},
+            "next_rows": {"fm": {"forward": {"ms": 0.1, "bytes": 1e6}, "backward": {"ms": 0.2, "bytes": 2e6}},
+                          "weight_grad": {"ms": 0.3, "bytes": 3e6},
+                          "backward_apply": {"sgd": {"ms": 3.0, "bytes": 4e6}}}}
+    bench.write_report(str(tmp_path / "r"), w, line, comp_ms, comp_bytes, [c], [[3, 1]], 1000.0)
+    doc = json.loads((tmp_path / "r.json").read_text())
+    names = [r["component"] for r in doc["components"]]
+    assert names[:3] == ["step", "step/forward", "step/forward/fwd.prep"]
+    assert "step/next/fm.forward" in names and "step/next/backward_apply.sgd" in names
+    gather = doc["components"][names.index("step/forward/fwd.gather")]
+    assert gather["est_avg_bw_gbs"] == pytest.approx(6000.0)  # 6 GB in 1 ms
+    bwd = doc["components"][names.index("step/backward")]
+    assert bwd["latency_ms"] == pytest.approx(2.8) and bwd["est_avg_bw_gbs"] == pytest.approx(8e9 / 2.8e-3 / 1e9, abs=0.1)
+    assert doc["components"][0]["latency_ms"] == 4.0
+    assert "| fwd.gather |" in (tmp_path / "r.md").read_text().replace("&nbsp;", "")
