@@ -345,3 +345,28 @@ def apply_step(tables, batch: int, indices, offsets, grad_out, weights=None, mea
         else:
             out.append(torch.from_numpy(a))
     return out, st
+
+
+# ----------------------------------------------------------------------------- batch replication
+
+def replicate_kjt(indices, offsets, weights, num_tables: int, factor: int):
+    """The batch-size preprocessor (Sec. III): a captured batch of B bags per table,
+    replicated to factor * B bags per table in the same key-major layout. Bag
+    r * B + b of table t (r < factor) is bag b of table t. Plain loops over bags.
+    Returns (indices, offsets, weights or None) as numpy arrays."""
+    ind = _np(indices)
+    off = _np(offsets)
+    w = None if weights is None else _np(weights, np.float32)
+    T = num_tables
+    B = (off.shape[0] - 1) // T
+    out_ind, out_w, out_off = [], [], [0]
+    for t in range(T):
+        for r in range(factor):
+            for b in range(B):
+                s, e = int(off[t * B + b]), int(off[t * B + b + 1])
+                out_ind.extend(ind[s:e].tolist())
+                if w is not None:
+                    out_w.extend(w[s:e].tolist())
+                out_off.append(out_off[-1] + (e - s))
+    return (np.array(out_ind, dtype=ind.dtype), np.array(out_off, dtype=off.dtype),
+            None if w is None else np.array(out_w, dtype=np.float32))
