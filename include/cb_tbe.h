@@ -216,6 +216,24 @@ cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int6
                              const void* offsets, const float* grad_out, float* grad_weights,
                              cudaStream_t stream);
 
+/* Batch-size preprocessor (Component Benchmark, Sec. III: a batch captured at a
+ * small size is replicated to the production batch size, keeping the input
+ * distribution). Input: a key-major batch of `batch` bags per table over
+ * `num_tables` tables (indices [num_indices], offsets [T*batch + 1], optional
+ * per-sample weights [num_indices]), all device memory of idx_dtype / fp32.
+ * Output: factor * batch bags per table, bag r*batch + b of table t (r <
+ * factor) being bag b of table t:
+ *   out_indices  device [factor * num_indices]
+ *   out_offsets  device [T * factor * batch + 1]
+ *   out_weights  device [factor * num_indices], or NULL when the input has none
+ * No handle, no allocation; invalid offsets are clamped (the output then has
+ * no meaning but every access stays in bounds). CB_ERR_INVALID_ARG for null
+ * buffers, factor < 1, or more than 2^31 output bags. */
+cb_status cb_kjt_replicate(const void* indices, const void* offsets, const float* per_sample_weights,
+                           cb_index_dtype idx_dtype, int32_t num_tables, int32_t batch,
+                           int64_t num_indices, int32_t factor, void* out_indices, void* out_offsets,
+                           float* out_weights, cudaStream_t stream);
+
 /* Releases the workspace and the handle (synchronises its last stream). */
 void cb_tbe_destroy(cb_tbe* h);
 

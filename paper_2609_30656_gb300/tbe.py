@@ -30,7 +30,7 @@ EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
            "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad",
-           "cb_tbe_backward_apply")
+           "cb_tbe_backward_apply", "cb_kjt_replicate")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -82,11 +82,12 @@ def load_library() -> ctypes.CDLL:
     lib.cb_tbe_weight_grad.argtypes = [p, i32, p, i64, p, p, p, p]
     lib.cb_tbe_backward_apply.argtypes = [p, i32, p, i64, p, p, p, ctypes.c_int, ctypes.c_float,
                                           ctypes.c_float, p, p]
+    lib.cb_kjt_replicate.argtypes = [p, p, p, ctypes.c_int, i32, i32, i64, i32, p, p, p, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
                  "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward",
-                 "cb_tbe_weight_grad", "cb_tbe_backward_apply"):
+                 "cb_tbe_weight_grad", "cb_tbe_backward_apply", "cb_kjt_replicate"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -365,3 +366,31 @@ def fm_backward(y: torch.Tensor, grad_fm: torch.Tensor, num_fields: int,
         _check(lib.cb_fm_backward(_ptr(y), _ptr(grad_fm), B, num_fields, D, stride, _ptr(out),
                                   stream), "cb_fm_backward")
     return out
+
+
+# ----------------------------------------------------------------------------- batch replication
+
+def replicate_batch(indices: torch.Tensor, offsets: torch.Tensor, weights: torch.Tensor | None,
+                    num_tables: int, factor: int):
+    """A captured batch replicated to factor x its bags per table (cb_kjt_replicate):
+    bag r * B + b of table t is bag b of table t. Returns device tensors
+    (indices, offsets, weights or None)."""
+    lib = load_library()
+    if indices.device.type != "cuda" or offsets.device != indices.device:
+        raise ValueError("indices and offsets must be CUDA tensors on one device")
+    if indices.dtype != offsets.dtype or indices.dtype not in _IDX:
+        raise ValueError("indices and offsets must both be int32 or both int64")
+    if num_tables < 1 or (offsets.numel() - 1) % num_tables:
+        raise ValueError("offsets must have num_tables * B + 1 entries")
+    B = (offsets.numel() - 1) // num_tables
+    ind, off = indices.contiguous(), offsets.contiguous()
+    w = None if weights is None else weights.to(indices.device, torch.float32).contiguous()
+    out_ind = torch.empty(factor * ind.numel(), dtype=ind.dtype, device=ind.device)
+    out_off = torch.empty(num_tables * factor * B + 1, dtype=off.dtype, device=ind.device)
+    out_w = None if w is None else torch.empty(factor * ind.numel(), dtype=torch.float32, device=ind.device)
+    with torch.cuda.device(ind.device):
+        stream = ctypes.c_void_p(torch.cuda.current_stream(ind.device).cuda_stream)
+        _check(lib.cb_kjt_replicate(_ptr(ind), _ptr(off), _ptr(w), _IDX[ind.dtype], num_tables, B,
+                                    ind.numel(), factor, _ptr(out_ind), _ptr(out_off), _ptr(out_w),
+                                    stream), "cb_kjt_replicate")
+    return out_ind, out_off, out_w

@@ -13,7 +13,7 @@ def _declared_functions():
     with open(os.path.join(ROOT, "include", "cb_tbe.h")) as f:
         text = f.read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(cb_(?:tbe|fm)_\w+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(cb_(?:tbe|fm|kjt)_\w+)\s*\(", text)))
 
 
 @pytest.fixture(scope="module")
@@ -73,6 +73,8 @@ def test_host_side_argument_errors_return_before_any_gpu_work(lib):
     assert lib.cb_fm_backward(None, None, 0, 0, 8, 0, None, None) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_fm_backward(None, None, 4, 2, 8, 12, None, None) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_fm_forward(None, 0, 2, 8, 16, None, None) == tbe.CB_OK  # nothing to do
+    # batch replication: factor < 1, null offsets
+    assert lib.cb_kjt_replicate(None, None, None, 1, 2, 4, 0, 2, None, None, None, None) == tbe.CB_ERR_INVALID_ARG
     # weight gradient and the fused optimizer step on a null handle
     assert lib.cb_tbe_weight_grad(None, 1, None, 0, None, None, None, None) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_tbe_backward_apply(None, 1, None, 0, None, None, None, 0, 0.1, 0.0, None,
