@@ -396,6 +396,9 @@ def run_ours(args):
         if len(set(w.dims)) == 1:
             nxt["fm"] = run_fm(w, out, flush, dev, peak)
         nxt["weight_grad"] = run_weight_grad(m, batches[0], grads_out[0], counts[0], flush, peak)
+        if all(d % 8 == 0 for d in w.dims):
+            nxt["mixed_precision_bf16"] = run_mixed_precision(w, tables, batches[0], grads_out[0], counts[0],
+                                                              uniq_tables[0], flush, peak)
         # last: it writes the tables
         nxt["backward_apply"] = run_backward_apply(m, w, batches[0], grads_out[0], counts[0],
                                                    uniq_tables[0], flush, peak, dev)
@@ -515,6 +518,51 @@ def run_weight_grad(m, b, go, c, flush, peak):
             "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes,
             "note": "algorithmic bytes count each lookup's row and grad_out slice; "
                     "repeated rows and a table's grad_out slice are largely served by L2"}
+
+
+def run_mixed_precision(w, tables, b, go, c, uniq, flush, peak):
+    """Forward and backward of one batch with the pooled output and grad_out in
+    bf16 (a second handle over the same tables, CB_OUT_BF16)."""
+    from paper_2609_30656_gb300 import tbe
+    m = tbe.TBE(tables, pooling="mean" if w.mean else "sum", out_dtype=torch.bfloat16)
+    go16 = go.to(torch.bfloat16)
+    out = torch.empty(w.batch, w.sum_dims, dtype=torch.bfloat16, device=go.device)
+    probe = m.alloc_grad(0, 0, size_only=True)
+    m.backward_into(probe, b.indices, b.offsets, go16, b.weights)
+    g = m.alloc_grad(probe.num_unique, probe.num_floats)
+    res = {}
+    for name in ("forward", "backward"):
+        def call():
+            if name == "forward":
+                m.forward(b.indices, b.offsets, b.weights, out=out)
+            else:
+                m.backward_into(g, b.indices, b.offsets, go16, b.weights)
+        for _ in range(2):
+            call()
+        torch.cuda.synchronize()
+        reps = 5
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for a, e in ev:
+            flush.zero_()
+            a.record()
+            call()
+            e.record()
+        torch.cuda.synchronize()
+        ms = statistics.mean(a.elapsed_time(e) for a, e in ev)
+        if name == "forward":
+            f = metrics.forward_bytes(c)
+            nbytes = f["total"] - f["output"] // 2  # bf16 output
+        else:
+            bb = metrics.backward_bytes(c, uniq)
+            nbytes = bb["total"] - bb["grad_gather"] // 2  # bf16 grad_out slices
+        res[name] = {"ms": round(ms, 4), "alg_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
+                     "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes}
+    if m.get_error() != 0:
+        raise RuntimeError("device-side error in the mixed-precision run")
+    m.close()
+    del g, out, go16
+    return res
 
 
 def run_backward_apply(m, w, b, go, c, uniq, flush, peak, dev):

@@ -64,6 +64,13 @@ typedef enum { CB_I32 = 0, CB_I64 = 1 } cb_index_dtype;
 /* Flags for cb_tbe_create. */
 #define CB_VALIDATE 0x1u  /* check offsets on device; synchronise and return errors */
 #define CB_TIMING   0x2u  /* record per-component CUDA events (cb_tbe_last_timings) */
+/* Mixed precision (the paper's mixed-precision preprocessor, Sec. III): the
+ * pooled output is written in fp16 / bf16 (the fp32 sums rounded to nearest
+ * even), and the backward, the weight gradient and the fused optimizer step take
+ * grad_out in the same type (summed in fp32; gradients stay fp32). At most one of
+ * the two; every table's dim must then be a multiple of 8. Default: fp32. */
+#define CB_OUT_F16  0x4u
+#define CB_OUT_BF16 0x8u
 /* Test hook: the first radix pass's tile 1 waits on a status word that nothing
  * writes, so its bounded wait runs out and the call reports CB_ERR_TIMEOUT. */
 #define CB_DEBUG_FORCE_LOOKBACK_TIMEOUT 0x100u
@@ -100,10 +107,11 @@ cb_status cb_tbe_reserve(cb_tbe* h, int32_t batch, int64_t num_indices);
  *   num_indices  n >= 0 (must equal offsets[T*B])
  *   offsets      device [T*B + 1], idx_dtype, key-major, non-decreasing, from 0
  *   per_sample_weights  device fp32 [n] or NULL
- *   out          device fp32 [B, sum of dims], row-major, 16-byte aligned;
+ *   out          device [B, sum of dims] of the output type (fp32; fp16 / bf16
+ *                under CB_OUT_F16 / CB_OUT_BF16), row-major, 16-byte aligned;
  *                every element is written. */
 cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
-                         const void* offsets, const float* per_sample_weights, float* out,
+                         const void* offsets, const float* per_sample_weights, void* out,
                          cudaStream_t stream);
 
 /* Forward without a handle and without allocating (the paper has no
@@ -152,13 +160,14 @@ typedef struct {
  *                       w_i * s_b(i) * grad_out[b(i), Doff_t : Doff_t + D_t]
  * computed by an on-device stable radix sort of (row id, lookup) pairs, a
  * run-length pass and a segmented reduction. Arguments as in cb_tbe_forward;
- * grad_out is device fp32 [B, sum of dims], 16-byte aligned. When U > cap_rows
+ * grad_out is device [B, sum of dims] of the output type (fp32 unless mixed
+ * precision), 16-byte aligned; gradients are fp32. When U > cap_rows
  * or F > cap_floats nothing is written to unique_ids / grad_offsets / grads,
  * num_unique and num_floats still hold the needed sizes, and the error is
  * CB_ERR_CAPACITY (returned now under CB_VALIDATE, else by cb_tbe_get_error). */
 cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
                           const void* offsets, const float* per_sample_weights,
-                          const float* grad_out, cb_sparse_grad* g, cudaStream_t stream);
+                          const void* grad_out, cb_sparse_grad* g, cudaStream_t stream);
 
 /* Synchronises the stream of the last call, returns the sticky device-side
  * error (CB_OK if none) and clears it. */
@@ -201,7 +210,7 @@ const char* cb_tbe_status_string(cb_status s);
 typedef enum { CB_OPT_SGD = 0, CB_OPT_ROWWISE_ADAGRAD = 1 } cb_optimizer;
 cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
                                 const void* offsets, const float* per_sample_weights,
-                                const float* grad_out, cb_optimizer kind, float lr, float eps,
+                                const void* grad_out, cb_optimizer kind, float lr, float eps,
                                 float* const* state, cudaStream_t stream);
 
 /* Gradient with respect to the per-sample weights (not in the paper; the
@@ -209,11 +218,12 @@ cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, i
  *   grad_weights[i] = s_b * sum_j grad_out[b, Doff_t + j] * E_t[indices[i], j]
  * for lookup i of bag (t, b), s_b = 1/L (mean pooling) or 1 (sum). The weights
  * themselves are not needed. Same batch, indices, num_indices and offsets as
- * cb_tbe_forward; grad_out device fp32 [B, sum of dims], 16-byte aligned;
+ * cb_tbe_forward; grad_out device [B, sum of dims] of the output type,
+ * 16-byte aligned;
  * grad_weights device fp32 [num_indices], every element written (0 for an
  * out-of-range index, which also sets CB_ERR_INDEX_OOB). Deterministic. */
 cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
-                             const void* offsets, const float* grad_out, float* grad_weights,
+                             const void* offsets, const void* grad_out, float* grad_weights,
                              cudaStream_t stream);
 
 /* Batch-size preprocessor (Component Benchmark, Sec. III: a batch captured at a

@@ -92,6 +92,7 @@ struct Workspace {
 
 struct cb_tbe {
     int device = 0;
+    int out_dtype = CB_F32;  // pooled output and grad_out: fp32, or fp16 / bf16 (mixed precision)
     int num_sms = 1;
     int32_t T = 0;
     int mode = CB_POOL_SUM;
@@ -226,6 +227,7 @@ Problem make_problem(const cb_tbe* h, int32_t B, const void* indices, int64_t n,
     P.is32 = h->is32;
     P.mean = h->mode == CB_POOL_MEAN;
     P.dmax = h->dmax;
+    P.out_dtype = h->out_dtype;
     return P;
 }
 
@@ -277,7 +279,7 @@ struct ApplyArgs {
 // The backward: into the caller's sparse-gradient buffers (g), or, with an
 // optimizer step (a), into the tables themselves.
 cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
-                        const void* offsets, const float* per_sample_weights, const float* grad_out,
+                        const void* offsets, const float* per_sample_weights, const void* grad_out,
                         cb_sparse_grad* g, const ApplyArgs* a, cudaStream_t stream) {
     cb_status st = check_common(h, batch, indices, num_indices, offsets);
     if (st != CB_OK) return st;
@@ -421,12 +423,8 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     // (5) segmented reduce, (6) fix-up of runs split across chunks
     if (reduce) {
         for (size_t c = 0; c < h->bwd_classes.size(); ++c) {
-            if (a)
-                launch_bwd_reduce_apply(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl,
-                                        h->bwd_classes[c].gc, packed, bound, h->num_sms, stream);
-            else
-                launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl,
-                                  h->bwd_classes[c].gc, packed, bound, h->num_sms, stream);
+            launch_bwd_reduce(P, Q, O, grad_out, static_cast<int>(c), h->bwd_classes[c].vpl, h->bwd_classes[c].gc,
+                              packed, a != nullptr, bound, h->num_sms, stream);
             h->launches += 1;
         }
         launch_bwd_fixup(P, Q, O, bound, h->num_sms, stream);
@@ -475,6 +473,12 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     h->mode = mode;
     h->is32 = idx_dtype == CB_I32;
     h->flags = flags;
+    if ((flags & CB_OUT_F16) && (flags & CB_OUT_BF16)) {
+        delete h;
+        return CB_ERR_INVALID_ARG;
+    }
+    h->out_dtype = (flags & CB_OUT_F16) ? CB_F16 : ((flags & CB_OUT_BF16) ? CB_BF16 : CB_F32);
+    const int out_eb = elem_bytes(h->out_dtype);
     int64_t row_base = 0, doff = 0;
     for (int32_t t = 0; t < num_tables; ++t) {
         const cb_table_desc& d = tables[t];
@@ -485,7 +489,8 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
             return CB_ERR_INVALID_ARG;
         }
         const int64_t row_bytes = static_cast<int64_t>(d.dim) * elem_bytes(d.dtype);
-        if (row_bytes % 16 != 0 || row_bytes > 2048) {
+        // grad_out rows of each table (the output's type) are whole 16-byte vectors too
+        if (row_bytes % 16 != 0 || row_bytes > 2048 || (static_cast<int64_t>(d.dim) * out_eb) % 16 != 0) {
             delete h;
             return CB_ERR_INVALID_ARG;
         }
@@ -498,7 +503,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
         td.dtype = d.dtype;
         td.row_vecs = static_cast<int32_t>(row_bytes / 16);
         lane_split(td.row_vecs, &td.lanes, &td.groups);
-        td.grad_vecs = d.dim / 4;
+        td.grad_vecs = d.dim * out_eb / 16;  // grad_out row, in the output's type
         lane_split(td.grad_vecs, &td.grad_lanes, &td.grad_groups);
         row_base += d.rows;
         doff += d.dim;
@@ -520,7 +525,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
     h->passes = (bits + 7) / 8;
 
     // Kernel classes: forward by (storage dtype, vectors per lane), backward by
-    // vectors per lane of the fp32 gradient row.
+    // vectors per lane of the grad_out row (fp32, or the mixed-precision type).
     for (int32_t t = 0; t < num_tables; ++t) {
         TableDev& td = h->tables[t];
         const int fv = vpl_for(td.row_vecs), bv = vpl_for(td.grad_vecs);
@@ -536,7 +541,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
             return static_cast<int>(cls.size() - 1);
         };
         td.fwd_class = put(h->fwd_classes, td.dtype, fv, fg);
-        td.bwd_class = put(h->bwd_classes, CB_F32, bv, bg);
+        td.bwd_class = put(h->bwd_classes, h->out_dtype, bv, bg);
     }
 
     if (cudaGetDevice(&h->device) != cudaSuccess ||
@@ -619,7 +624,7 @@ cb_status cb_tbe_reserve(cb_tbe* h, int32_t batch, int64_t num_indices) {
 }
 
 cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
-                         const void* offsets, const float* per_sample_weights, float* out,
+                         const void* offsets, const float* per_sample_weights, void* out,
                          cudaStream_t stream) {
     cb_status st = check_common(h, batch, indices, num_indices, offsets);
     if (st != CB_OK) return st;
@@ -636,7 +641,8 @@ cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t 
         h->launches += 1;
     }
     if (n == 0) {
-        if (cudaMemsetAsync(out, 0, sizeof(float) * batch * h->sum_d, stream) != cudaSuccess)
+        if (cudaMemsetAsync(out, 0, static_cast<size_t>(elem_bytes(h->out_dtype)) * batch * h->sum_d, stream) !=
+            cudaSuccess)
             return CB_ERR_CUDA;
         return finish_call(h, stream);
     }
@@ -663,7 +669,7 @@ cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t 
 }
 
 cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
-                             const void* offsets, const float* grad_out, float* grad_weights,
+                             const void* offsets, const void* grad_out, float* grad_weights,
                              cudaStream_t stream) {
     cb_status st = check_common(h, batch, indices, num_indices, offsets);
     if (st != CB_OK) return st;
@@ -699,7 +705,7 @@ cb_status cb_tbe_weight_grad(cb_tbe* h, int32_t batch, const void* indices, int6
 
 cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
                           const void* offsets, const float* per_sample_weights,
-                          const float* grad_out, cb_sparse_grad* g, cudaStream_t stream) {
+                          const void* grad_out, cb_sparse_grad* g, cudaStream_t stream) {
     if (!h) return CB_ERR_INVALID_ARG;
     if (!g || !g->table_offsets || !g->num_unique || !g->num_floats) return CB_ERR_INVALID_ARG;
     if (g->grads && (!g->unique_ids || !g->grad_offsets || g->cap_rows < 0 || g->cap_floats < 0 ||
@@ -711,7 +717,7 @@ cb_status cb_tbe_backward(cb_tbe* h, int32_t batch, const void* indices, int64_t
 
 cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, int64_t num_indices,
                                 const void* offsets, const float* per_sample_weights,
-                                const float* grad_out, cb_optimizer kind, float lr, float eps,
+                                const void* grad_out, cb_optimizer kind, float lr, float eps,
                                 float* const* state, cudaStream_t stream) {
     if (!h) return CB_ERR_INVALID_ARG;
     if (kind != CB_OPT_SGD && kind != CB_OPT_ROWWISE_ADAGRAD) return CB_ERR_INVALID_ARG;

@@ -186,6 +186,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
     P.is32 = idx_dtype == CB_I32;
     P.mean = mode == CB_POOL_MEAN;
     P.dmax = dmax;
+    P.out_dtype = CB_F32;
     int num_sms = 1;
     cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, device);
     launch_validate_offsets(P, num_sms, stream);

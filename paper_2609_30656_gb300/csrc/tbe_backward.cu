@@ -344,10 +344,18 @@ void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s) {
     bwd_finalize_kernel<<<1, 1024, 0, s>>>(P, O);
 }
 
-void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
-                       int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
+void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out, int cls,
+                       int vpl, int gc, bool packed, bool apply, int64_t chunk_bound, int num_sms,
                        cudaStream_t s) {
-    launch_bwd_reduce_t<false>(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
+    if (P.out_dtype == CB_F16) {
+        launch_bwd_reduce_f16(P, Q, O, grad_out, cls, vpl, gc, packed, apply, chunk_bound, num_sms, s);
+    } else if (P.out_dtype == CB_BF16) {
+        launch_bwd_reduce_bf16(P, Q, O, grad_out, cls, vpl, gc, packed, apply, chunk_bound, num_sms, s);
+    } else if (apply) {
+        launch_bwd_reduce_f32_apply(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
+    } else {
+        launch_bwd_reduce_t<CB_F32, false>(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
+    }
 }
 
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,

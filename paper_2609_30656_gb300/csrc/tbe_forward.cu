@@ -10,7 +10,7 @@ namespace cbtbe {
 // scans 32 chunks at a time for tails (rare once boundaries snap to bag ends).
 __global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(const __grid_constant__ Problem P,
                                                                  const __grid_constant__ Plan Q,
-                                                                 float* out) {
+                                                                 void* out) {
     const int lane = threadIdx.x & 31;
     const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     for (int64_t base = warp_id_global() * 32; base < total; base += warps_in_grid() * 32) {
@@ -25,33 +25,32 @@ __global__ void __launch_bounds__(kWarpThreads) fwd_fixup_kernel(const __grid_co
             const int64_t e = load_index(P.offsets, bag + 1, P.is32);
             const int64_t m = pieces_after(Q, j, e, total);
             const double L = (P.mean && e > s) ? static_cast<double>(e - s) : 0.0;
-            float* dst = out + (bag - static_cast<int64_t>(t) * P.B) * P.sum_d + td.doff;
+            const int64_t col0 = (bag - static_cast<int64_t>(t) * P.B) * P.sum_d + td.doff;
             combine_pieces(Q, j, m, td.dim, P.dmax, lane, [&](int x0, double (&acc)[4]) {
                 if (L > 0.0)
                     for (int x = 0; x < 4; ++x) acc[x] /= L;
-                *reinterpret_cast<float4*>(dst + x0) =
-                    make_float4(static_cast<float>(acc[0]), static_cast<float>(acc[1]),
-                                static_cast<float>(acc[2]), static_cast<float>(acc[3]));
+                store_out4(out, col0 + x0, static_cast<float>(acc[0]), static_cast<float>(acc[1]),
+                           static_cast<float>(acc[2]), static_cast<float>(acc[3]), P.out_dtype);
             });
         }
     }
 }
 
-void launch_fwd_gather_f32(const Problem&, const Plan&, float*, int, int, int, int64_t, int,
+void launch_fwd_gather_f32(const Problem&, const Plan&, void*, int, int, int, int64_t, int,
                            cudaStream_t);
-void launch_fwd_gather_f16(const Problem&, const Plan&, float*, int, int, int, int64_t, int,
+void launch_fwd_gather_f16(const Problem&, const Plan&, void*, int, int, int, int64_t, int,
                            cudaStream_t);
-void launch_fwd_gather_bf16(const Problem&, const Plan&, float*, int, int, int, int64_t, int,
+void launch_fwd_gather_bf16(const Problem&, const Plan&, void*, int, int, int, int64_t, int,
                             cudaStream_t);
 
-void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,
+void launch_fwd_gather(const Problem& P, const Plan& Q, void* out, int cls, int dtype, int vpl,
                        int gc, int64_t chunk_bound, int num_sms, cudaStream_t s) {
     if (dtype == CB_F32) launch_fwd_gather_f32(P, Q, out, cls, vpl, gc, chunk_bound, num_sms, s);
     else if (dtype == CB_F16) launch_fwd_gather_f16(P, Q, out, cls, vpl, gc, chunk_bound, num_sms, s);
     else launch_fwd_gather_bf16(P, Q, out, cls, vpl, gc, chunk_bound, num_sms, s);
 }
 
-void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
+void launch_fwd_fixup(const Problem& P, const Plan& Q, void* out, int64_t chunk_bound,
                       int num_sms, cudaStream_t s) {
     const int64_t need = (chunk_bound + kWarpThreads - 1) / kWarpThreads;  // 32 chunks per warp
     const int grid = static_cast<int>(max64(1, min64(need, static_cast<int64_t>(num_sms) * 8)));

@@ -23,12 +23,13 @@ struct FwdPolicy {
     static constexpr int kVpl = VPL;
     static constexpr int kUnroll = CB_WALK_ROWS / VPL > 0 ? CB_WALK_ROWS / VPL : 1;
     static constexpr bool kWeighted = WEIGHTED;
+    static constexpr bool kTwoLevel = DT == CB_F32;  // half rows: one fp32 level (registers)
     static constexpr bool kUnrollGroups = CB_WALK_UNROLL_GROUPS;
     static constexpr bool kFastBatch = CB_WALK_FAST_BATCH;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;
-    float* out;
+    void* out;         // [B, sum D] of P.out_dtype
     const uint4* base;  // the table
     int64_t rows;
     uint32_t stride;    // 16-byte vectors per row
@@ -66,29 +67,37 @@ struct FwdPolicy {
     // An empty bag pools to zeros (one vector per lane).
     __device__ __forceinline__ void put_empty(int32_t bag, int v, bool group0) const {
         if (!group0) return;
-        float4* d4 = reinterpret_cast<float4*>(out + static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff +
-                                               v * kElems);
+        const int64_t col = static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff + v * kElems;
 #pragma unroll
-        for (int x = 0; x < kElems / 4; ++x) d4[x] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int x = 0; x < kElems / 4; ++x) store_out4(out, col + 4 * x, 0.f, 0.f, 0.f, 0.f, P.out_dtype);
     }
     __device__ __forceinline__ void emit(int32_t bag, int32_t L, bool started, bool ends,
                                          float (&tot)[VPL][kElems], int v, bool group0) const {
         if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = bag;
         if (!group0) return;
-        float* dst;
-        float scale = 0.f;
         if (started && ends) {
-            dst = out + static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff;
-            if (P.mean && L > 0) scale = static_cast<float>(L);
-        } else {
-            dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
-        }
-        if (scale > 0.f) {  // mean pooling of a complete, non-empty bag
+            // A complete bag: the pooled row, in the output's type.
+            if (P.mean && L > 0) {
+                const float scale = static_cast<float>(L);
 #pragma unroll
-            for (int k = 0; k < VPL; ++k)
+                for (int k = 0; k < VPL; ++k)
 #pragma unroll
-                for (int x = 0; x < kElems; ++x) tot[k][x] = tot[k][x] / scale;
+                    for (int x = 0; x < kElems; ++x) tot[k][x] = tot[k][x] / scale;
+            }
+            const int64_t col0 = static_cast<int64_t>(bag - bag_lo) * P.sum_d + doff;
+#pragma unroll
+            for (int k = 0; k < VPL; ++k) {
+                const int vec = v + 32 * k;
+                if (vec >= row_vecs) continue;
+#pragma unroll
+                for (int x = 0; x < kElems / 4; ++x)
+                    store_out4(out, col0 + vec * kElems + 4 * x, tot[k][4 * x], tot[k][4 * x + 1],
+                               tot[k][4 * x + 2], tot[k][4 * x + 3], P.out_dtype);
+            }
+            return;
         }
+        // A piece of a bag split across chunks: fp32, for the fix-up.
+        float* dst = (started ? Q.carry_tail : Q.carry_head) + static_cast<int64_t>(chunk) * P.dmax;
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
             const int vec = v + 32 * k;
@@ -103,7 +112,7 @@ struct FwdPolicy {
 
 template <int DT, int VPL, bool WEIGHTED, int GC>
 __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
-    fwd_gather_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q, float* out,
+    fwd_gather_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q, void* out,
                       int cls) {
     const int lane = threadIdx.x & 31;
     const int64_t cb = Q.class_chunk_base[cls];
@@ -151,7 +160,7 @@ static int gather_grid(int num_sms) {
 }
 
 template <int DT, int VPL, int GC>
-static void launch_gather_layout(const Problem& P, const Plan& Q, float* out, int cls,
+static void launch_gather_layout(const Problem& P, const Plan& Q, void* out, int cls,
                                  int64_t chunk_bound, int num_sms, cudaStream_t s) {
     const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
     if (P.weights) {
@@ -166,7 +175,7 @@ static void launch_gather_layout(const Problem& P, const Plan& Q, float* out, in
 // Row layouts compiled for: (vectors per lane, rows per step) =
 // (1, 1|2|4|8), (2, 1), (4, 1), and (1, run-time) for odd row sizes.
 template <int DT>
-void launch_gather_dtype(const Problem& P, const Plan& Q, float* out, int cls, int vpl, int gc,
+void launch_gather_dtype(const Problem& P, const Plan& Q, void* out, int cls, int vpl, int gc,
                          int64_t chunk_bound, int num_sms, cudaStream_t s) {
 #define CB_CASE(V, G)                                                                \
     if (vpl == V && gc == G) {                                                        \

@@ -18,6 +18,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
+#include <cuda_bf16.h>
 #include <type_traits>
 
 #include "cb_tbe.h"
@@ -101,6 +102,7 @@ struct Problem {
     int32_t is32;
     int32_t mean;
     int32_t dmax;  // largest dim (row stride of the carry buffers)
+    int32_t out_dtype;  // cb_dtype of the pooled output and of grad_out
 };
 
 struct Plan {
@@ -228,6 +230,31 @@ __device__ __forceinline__ void unpack<CB_BF16>(const uint4& r, float (&f)[8]) {
     }
 }
 
+// ---------------------------------------------------------------- output rows
+
+// Four consecutive columns of an output row, stored as fp32 or rounded to
+// fp16 / bf16 (round to nearest even).
+__device__ __forceinline__ void store_out4(void* row, int64_t col, float a, float b, float c, float d,
+                                           int dtype) {
+    if (dtype == CB_F32) {
+        *reinterpret_cast<float4*>(static_cast<float*>(row) + col) = make_float4(a, b, c, d);
+        return;
+    }
+    uint2 w;
+    if (dtype == CB_F16) {
+        const __half2 lo = __floats2half2_rn(a, b), hi = __floats2half2_rn(c, d);
+        memcpy(&w.x, &lo, 4);
+        memcpy(&w.y, &hi, 4);
+    } else {
+        const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+        memcpy(&w.x, &lo, 4);
+        memcpy(&w.y, &hi, 4);
+    }
+    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(row) + col) = w;
+}
+
+__host__ __device__ __forceinline__ int dtype_bytes(int dtype) { return dtype == CB_F32 ? 4 : 2; }
+
 // ---------------------------------------------------------------- accumulation
 
 // acc += w * row (WEIGHTED) or acc += row. Half-precision rows use the
@@ -340,7 +367,7 @@ __device__ __forceinline__ void walk_chunk(Pol& pol, const ChunkCtx& c, const ui
     // fp32 rows (tables or gradients) sum in two levels (see the fold below);
     // half-precision rows, whose tolerance is far looser, use one level, which
     // frees registers for occupancy.
-    constexpr bool kTwoLevel = Pol::kDtype == CB_F32;
+    constexpr bool kTwoLevel = Pol::kTwoLevel;
     float ain[VPL][E], aout[VPL][kTwoLevel ? E : 1];
 #pragma unroll
     for (int k = 0; k < VPL; ++k) {
@@ -519,7 +546,7 @@ __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uin
     constexpr uint32_t kGroupMask = kGroupItems == 32 ? kFull : (1u << kGroupItems) - 1u;
     constexpr uint32_t kStepMask = (1u << G) - 1u;
     constexpr bool W = Pol::kWeighted;
-    constexpr bool kTwoLevel = Pol::kDtype == CB_F32;
+    constexpr bool kTwoLevel = Pol::kTwoLevel;
     constexpr int kGroupUnroll = Pol::kUnrollGroups ? 32 / kGroupItems : 1;
     const int g = lane / V;
     const int v = lane - g * V;

@@ -74,9 +74,9 @@ void launch_validate_offsets(const Problem& P, int num_sms, cudaStream_t s);
 void launch_plan(const Problem& P, const Plan& Q, int mode, const uint32_t* seg_start,
                  const int64_t* num_unique, int num_sms, bool tables_too, cudaStream_t s);
 
-void launch_fwd_gather(const Problem& P, const Plan& Q, float* out, int cls, int dtype, int vpl,
+void launch_fwd_gather(const Problem& P, const Plan& Q, void* out, int cls, int dtype, int vpl,
                        int gc, int64_t chunk_bound, int num_sms, cudaStream_t s);
-void launch_fwd_fixup(const Problem& P, const Plan& Q, float* out, int64_t chunk_bound,
+void launch_fwd_fixup(const Problem& P, const Plan& Q, void* out, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
 
 constexpr int64_t kSortTileKeys = 4096;
@@ -93,9 +93,20 @@ int64_t rle_num_tiles(int64_t n);
 void launch_rle(const uint32_t* keys, int64_t n, int64_t* tile_heads, int64_t* tile_base,
                 int64_t* num_unique, uint32_t* uniq, uint32_t* seg_start, cudaStream_t s);
 void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s);
-void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
-                       int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
+// The segmented reduce (apply: with the optimizer step fused), dispatched on
+// the grad_out type P.out_dtype; one translation unit per type.
+void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out, int cls,
+                       int vpl, int gc, bool packed, bool apply, int64_t chunk_bound, int num_sms,
                        cudaStream_t s);
+void launch_bwd_reduce_f32_apply(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out,
+                                 int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
+                                 cudaStream_t s);
+void launch_bwd_reduce_f16(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out, int cls,
+                           int vpl, int gc, bool packed, bool apply, int64_t chunk_bound, int num_sms,
+                           cudaStream_t s);
+void launch_bwd_reduce_bf16(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out, int cls,
+                            int vpl, int gc, bool packed, bool apply, int64_t chunk_bound, int num_sms,
+                            cudaStream_t s);
 // Rows per warp step fixed at compile time for a row of `vecs` 16-byte vectors
 // spread as (lanes, groups), or 0 when the layout is only known at run time.
 inline int compile_time_groups(int vpl, int lanes, int groups) {
@@ -103,11 +114,8 @@ inline int compile_time_groups(int vpl, int lanes, int groups) {
     if (lanes * groups == 32 && (groups == 1 || groups == 2 || groups == 4 || groups == 8)) return groups;
     return 0;
 }
-void launch_weight_grad(const Problem& P, const Plan& Q, const float* grad_out, float* grad_w, int cls,
+void launch_weight_grad(const Problem& P, const Plan& Q, const void* grad_out, float* grad_w, int cls,
                         int dtype, int gc, int64_t chunk_bound, int num_sms, cudaStream_t s);
-void launch_bwd_reduce_apply(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
-                             int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
-                             cudaStream_t s);
 void launch_bwd_fixup(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,
                       int num_sms, cudaStream_t s);
 void launch_bwd_apply_split(const Problem& P, const Plan& Q, const BwdOut& O, int64_t chunk_bound,

@@ -10,6 +10,10 @@
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
 
+#ifndef CB_REDUCE_HALF_ROWS
+#define CB_REDUCE_HALF_ROWS 4  // rows in flight per lane for fp16 / bf16 grad_out
+#endif
+
 namespace cbtbe {
 
 template <class KernelT>
@@ -87,49 +91,54 @@ __device__ __forceinline__ float step_scale(const BwdOut& O, int t, int64_t row,
 // group 0 writes. Out of line: the walker ends runs in many places, and a copy
 // of the step in each of them overflowed the instruction cache (measured on
 // cfg5: fused SGD step 36.8 ms inline, 21 ms out of line).
-template <int VPL>
+template <int N>
 struct GradRow {
-    float4 v[VPL];
+    float4 v[N];   // four gradient columns each
+    int col[N];    // first column of each, or -1 past the row
 };
 
-template <int VPL>
+template <int N>
 __device__ __noinline__ void apply_row(const Problem& P, const BwdOut& O, int t, int32_t seg,
-                                       const GradRow<VPL> g, int v, bool group0) {
+                                       const GradRow<N> g, bool group0) {
     const TableDev& td = P.tables[t];
     const int64_t row = static_cast<int64_t>(__ldg(O.uniq + seg)) - td.row_base;
-    const int nv = td.dim / 4;
     float sq = 0.f;
 #pragma unroll
-    for (int k = 0; k < VPL; ++k)
-        if (group0 && v + 32 * k < nv)
+    for (int k = 0; k < N; ++k)
+        if (group0 && g.col[k] >= 0)
             sq += g.v[k].x * g.v[k].x + g.v[k].y * g.v[k].y + g.v[k].z * g.v[k].z + g.v[k].w * g.v[k].w;
     const float scale = step_scale(O, t, row, td.dim, sq);
     if (!group0) return;
 #pragma unroll
-    for (int k = 0; k < VPL; ++k)
-        if (v + 32 * k < nv) step_cols(td, row, 4 * (v + 32 * k), g.v[k], scale);
+    for (int k = 0; k < N; ++k)
+        if (g.col[k] >= 0) step_cols(td, row, g.col[k], g.v[k], scale);
 }
 
 // ---------------------------------------------------------------- (5) reduce
 
 // APPLY: the optimizer step is fused where a run's sum ends (compiled as its
 // own kernels, so the gradient-writing reduce carries none of its code).
-template <int VPL, bool PACKED, bool APPLY>
+template <int GO, int VPL, bool PACKED, bool APPLY>
 struct BwdPolicy {
-    static constexpr int kDtype = CB_F32;
-    static constexpr int kElems = 4;
+    static constexpr int kDtype = GO;  // grad_out storage: fp32, or fp16 / bf16 (mixed precision)
+    static constexpr int kElems = Storage<GO>::kElems;
+    static constexpr bool kTwoLevel = true;  // gradients keep the fp32 bound for every grad_out type
     static constexpr int kVpl = VPL;
-    static constexpr int kUnroll = CB_REDUCE_ROWS / VPL > 0 ? CB_REDUCE_ROWS / VPL : 1;
+    // Half grad_out rows (8 values per lane, usually 2 rows per warp step) take
+    // the forward's code shape: fewer rows in flight, one copy of the run-end
+    // code per batch.
+    static constexpr int kRows = GO == CB_F32 ? CB_REDUCE_ROWS : CB_REDUCE_HALF_ROWS;
+    static constexpr int kUnroll = kRows / VPL > 0 ? kRows / VPL : 1;
     static constexpr bool kWeighted = PACKED;
-    static constexpr bool kUnrollGroups = CB_REDUCE_UNROLL_GROUPS;
-    static constexpr bool kFastBatch = CB_REDUCE_FAST_BATCH;
+    static constexpr bool kUnrollGroups = GO == CB_F32 ? CB_REDUCE_UNROLL_GROUPS : false;
+    static constexpr bool kFastBatch = GO == CB_F32 ? CB_REDUCE_FAST_BATCH : true;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;
     const BwdOut& O;
     const uint4* base;  // grad_out + Doff_t, one row per bag of this table
     int64_t float_lo;   // first float of this table in grads
-    uint32_t stride;    // sum of dims / 4
+    uint32_t stride;    // 16-byte vectors per grad_out row
     int32_t chunk;
     int32_t bag_lo;
     int32_t seg_lo;     // first unique index of this table
@@ -171,20 +180,29 @@ struct BwdPolicy {
     }
     __device__ __forceinline__ void put_empty(int32_t, int, bool) const {}
     __device__ __forceinline__ void emit(int32_t seg, int32_t L, bool started, bool ends,
-                                         float (&tot)[VPL][4], int v, bool group0) const {
+                                         float (&tot)[VPL][kElems], int v, bool group0) const {
         if (started && (threadIdx.x & 31) == 0) seg_meta(seg);
         put(seg, L, started, ends, tot, v, group0);
     }
+    // Lane v of a row group holds vectors v + 32k of the grad_out row: columns
+    // [(v + 32k) * kElems, + kElems), written as fp32 gradients.
     __device__ __forceinline__ void put(int32_t seg, int32_t, bool started, bool ends,
-                                        float (&tot)[VPL][4], int v, bool group0) const {
+                                        float (&tot)[VPL][kElems], int v, bool group0) const {
         const int64_t fo = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
         if (started && !ends && (threadIdx.x & 31) == 0) Q.tail_owner[chunk] = seg;
         if constexpr (APPLY) {
             if (started && ends) {
-                GradRow<VPL> r;
+                GradRow<VPL * kElems / 4> r;
 #pragma unroll
-                for (int k = 0; k < VPL; ++k) r.v[k] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
-                apply_row<VPL>(P, O, table, seg, r, v, group0);
+                for (int k = 0; k < VPL; ++k)
+#pragma unroll
+                    for (int x = 0; x < kElems / 4; ++x) {
+                        const int col = (v + 32 * k) * kElems + 4 * x;
+                        r.v[k * (kElems / 4) + x] = make_float4(tot[k][4 * x], tot[k][4 * x + 1],
+                                                                tot[k][4 * x + 2], tot[k][4 * x + 3]);
+                        r.col[k * (kElems / 4) + x] = col < dim ? col : -1;
+                    }
+                apply_row<VPL * kElems / 4>(P, O, table, seg, r, group0);
                 return;
             }
         }
@@ -195,16 +213,20 @@ struct BwdPolicy {
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
             const int vec = v + 32 * k;
-            if (vec < dim / 4)
-                reinterpret_cast<float4*>(dst)[vec] = make_float4(tot[k][0], tot[k][1], tot[k][2], tot[k][3]);
+            if (vec * kElems < dim) {
+                float4* d4 = reinterpret_cast<float4*>(dst + vec * kElems);
+#pragma unroll
+                for (int x = 0; x < kElems / 4; ++x)
+                    d4[x] = make_float4(tot[k][4 * x], tot[k][4 * x + 1], tot[k][4 * x + 2], tot[k][4 * x + 3]);
+            }
         }
     }
 };
 
-template <int VPL, bool PACKED, int GC, bool APPLY>
+template <int GO, int VPL, bool PACKED, int GC, bool APPLY>
 __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
     bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
-                      const __grid_constant__ BwdOut O, const float* grad_out, int cls) {
+                      const __grid_constant__ BwdOut O, const void* grad_out, int cls) {
     if (*O.cap_fail) return;
     const int lane = threadIdx.x & 31;
     const int64_t cb = Q.class_chunk_base[cls];
@@ -213,10 +235,12 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];
-        BwdPolicy<VPL, PACKED, APPLY> pol{P, Q, O};
-        pol.base = reinterpret_cast<const uint4*>(grad_out + td.doff);
+        BwdPolicy<GO, VPL, PACKED, APPLY> pol{P, Q, O};
+        constexpr int eb = GO == CB_F32 ? 4 : 2;
+        pol.base = reinterpret_cast<const uint4*>(static_cast<const char*>(grad_out) +
+                                                  static_cast<int64_t>(td.doff) * eb);
         pol.float_lo = O.float_base[t];
-        pol.stride = static_cast<uint32_t>(P.sum_d / 4);
+        pol.stride = static_cast<uint32_t>(P.sum_d * eb / 16);
         pol.chunk = static_cast<int32_t>(j);
         pol.bag_lo = t * P.B;
         pol.seg_lo = static_cast<int32_t>(O.table_first[t]);
@@ -234,27 +258,28 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
         if (lane == 0) Q.tail_owner[j] = -1;
         if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
             __shared__ EndSlot slots[kWarpThreads / 32][32];
-            walk_rows<BwdPolicy<VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+            walk_rows<BwdPolicy<GO, VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
         } else {
-            walk_chunk<BwdPolicy<VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane);
+            walk_chunk<BwdPolicy<GO, VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane);
         }
     }
 }
 
-template <int VPL, bool PACKED, int GC, bool APPLY>
-static void launch_reduce_one(const Problem& P, const Plan& Q, const BwdOut& O, const float* go,
+template <int GO, int VPL, bool PACKED, int GC, bool APPLY>
+static void launch_reduce_one(const Problem& P, const Plan& Q, const BwdOut& O, const void* go,
                               int cls, int64_t chunk_bound, int num_sms, cudaStream_t s) {
-    static int cap = occupancy_grid(bwd_reduce_kernel<VPL, PACKED, GC, APPLY>, kWarpThreads, num_sms);
-    bwd_reduce_kernel<VPL, PACKED, GC, APPLY><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(P, Q, O, go, cls);
+    static int cap = occupancy_grid(bwd_reduce_kernel<GO, VPL, PACKED, GC, APPLY>, kWarpThreads, num_sms);
+    bwd_reduce_kernel<GO, VPL, PACKED, GC, APPLY><<<warp_grid(chunk_bound, cap), kWarpThreads, 0, s>>>(
+        P, Q, O, go, cls);
 }
 
-template <bool APPLY>
-void launch_bwd_reduce_t(const Problem& P, const Plan& Q, const BwdOut& O, const float* grad_out,
+template <int GO, bool APPLY>
+void launch_bwd_reduce_t(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out,
                          int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
                          cudaStream_t s) {
 #define CB_CASE(V, G, PK)                                                                \
     if (vpl == V && gc == G && packed == PK) {                                            \
-        launch_reduce_one<V, PK, G, APPLY>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s);    \
+        launch_reduce_one<GO, V, PK, G, APPLY>(P, Q, O, grad_out, cls, chunk_bound, num_sms, s); \
         return;                                                                          \
     }
     CB_CASE(1, 1, false) CB_CASE(1, 2, false) CB_CASE(1, 4, false) CB_CASE(1, 8, false)

@@ -12,8 +12,9 @@
 // window of bag ends; then G = 32 / V lookups per warp step (V lanes per stored
 // row, 16 bytes each), several steps' loads in flight, a dot product per lane
 // and a butterfly over the row's lanes. Consecutive lookups of one bag read the
-// same grad_out slice, which L1 serves. The dot products are summed in a fixed
-// order (deterministic).
+// same grad_out slice, which L1 serves. grad_out is fp32, or fp16 / bf16 when
+// the handle's output is (mixed precision). The dot products are summed in a
+// fixed order (deterministic).
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
 
@@ -22,16 +23,31 @@ namespace {
 
 constexpr int kWgradSteps = 4;  // warp steps whose loads are issued together
 
+// Four grad_out values at g (fp32, or fp16 / bf16 with mixed precision), widened.
+__device__ __forceinline__ float4 load_go4(const char* g, int go_dtype) {
+    if (go_dtype == CB_F32) return __ldg(reinterpret_cast<const float4*>(g));
+    const uint2 w = __ldg(reinterpret_cast<const uint2*>(g));
+    if (go_dtype == CB_BF16)
+        return make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xffff0000u),
+                           __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xffff0000u));
+    __half2 a, b;
+    memcpy(&a, &w.x, 4);
+    memcpy(&b, &w.y, 4);
+    const float2 fa = __half22float2(a), fb = __half22float2(b);
+    return make_float4(fa.x, fa.y, fb.x, fb.y);
+}
+
+// <row vector x, the E grad_out values at g>, g in bytes of the grad_out type.
 template <int DT>
-__device__ __forceinline__ float dot_row(const uint4& x, const float* g) {
+__device__ __forceinline__ float dot_row(const uint4& x, const char* g, int go_dtype) {
     constexpr int E = Storage<DT>::kElems;
     float f[E];
     unpack<DT>(x, f);
-    const float4* g4 = reinterpret_cast<const float4*>(g);
+    const int step = go_dtype == CB_F32 ? 16 : 8;
     float acc = 0.f;
 #pragma unroll
     for (int k = 0; k < E / 4; ++k) {
-        const float4 q = __ldg(g4 + k);
+        const float4 q = load_go4(g + k * step, go_dtype);
         acc = fmaf(q.x, f[4 * k], acc);
         acc = fmaf(q.y, f[4 * k + 1], acc);
         acc = fmaf(q.z, f[4 * k + 2], acc);
@@ -46,7 +62,7 @@ __device__ __forceinline__ float dot_row(const uint4& x, const float* g) {
 template <int DT, int GC>
 __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_constant__ Problem P,
                                                                    const __grid_constant__ Plan Q,
-                                                                   const float* grad_out, float* grad_w,
+                                                                   const void* grad_out, float* grad_w,
                                                                    int cls) {
     constexpr int E = Storage<DT>::kElems;
     constexpr int G = GC > 0 ? GC : 1;
@@ -63,7 +79,8 @@ __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_
         const int nvec = td.row_vecs;
         const int64_t k0 = ch.k0, k1 = ch.k0 + (ch.len & 0x7fffffffu);
         const int64_t bag_lo = static_cast<int64_t>(t) * P.B, bag_hi = bag_lo + P.B;
-        const float* go_base = grad_out + td.doff;
+        const int eb = dtype_bytes(P.out_dtype);
+        const char* go_base = static_cast<const char*>(grad_out) + static_cast<int64_t>(td.doff) * eb;
         BagWindow W = bag_window(P, ch.first, bag_hi, lane);
         for (int64_t base = k0; base < k1; base += 32) {
             const int64_t q = base + lane;
@@ -96,11 +113,12 @@ __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_
                     dot[u] = 0.f;
                     if (i >= nb || a == kInvalid) continue;
                     const uint4* rp = rows + static_cast<int64_t>(a) * nvec;
-                    const float* gp = go_base + go;
+                    const char* gp = go_base + go * eb;
                     if (GC > 0) {
-                        dot[u] = dot_row<DT>(__ldg(rp + v), gp + v * E);
+                        dot[u] = dot_row<DT>(__ldg(rp + v), gp + v * E * eb, P.out_dtype);
                     } else {
-                        for (int vec = v; vec < nvec; vec += 32) dot[u] += dot_row<DT>(__ldg(rp + vec), gp + vec * E);
+                        for (int vec = v; vec < nvec; vec += 32)
+                            dot[u] += dot_row<DT>(__ldg(rp + vec), gp + vec * E * eb, P.out_dtype);
                     }
                 }
 #pragma unroll
@@ -117,7 +135,7 @@ __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_
 }
 
 template <int DT, int GC>
-void launch_one(const Problem& P, const Plan& Q, const float* go, float* gw, int cls, int64_t chunk_bound,
+void launch_one(const Problem& P, const Plan& Q, const void* go, float* gw, int cls, int64_t chunk_bound,
                 int num_sms, cudaStream_t s) {
     static int per_sm = -1;
     if (per_sm < 0 && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, weight_grad_kernel<DT, GC>,
@@ -130,7 +148,7 @@ void launch_one(const Problem& P, const Plan& Q, const float* go, float* gw, int
 }
 
 template <int DT>
-void launch_dtype(const Problem& P, const Plan& Q, const float* go, float* gw, int cls, int gc,
+void launch_dtype(const Problem& P, const Plan& Q, const void* go, float* gw, int cls, int gc,
                   int64_t chunk_bound, int num_sms, cudaStream_t s) {
     switch (gc) {
         case 1: launch_one<DT, 1>(P, Q, go, gw, cls, chunk_bound, num_sms, s); break;
@@ -143,7 +161,7 @@ void launch_dtype(const Problem& P, const Plan& Q, const float* go, float* gw, i
 
 }  // namespace
 
-void launch_weight_grad(const Problem& P, const Plan& Q, const float* grad_out, float* grad_w, int cls,
+void launch_weight_grad(const Problem& P, const Plan& Q, const void* grad_out, float* grad_w, int cls,
                         int dtype, int gc, int64_t chunk_bound, int num_sms, cudaStream_t s) {
     if (dtype == CB_F32) launch_dtype<CB_F32>(P, Q, grad_out, grad_w, cls, gc, chunk_bound, num_sms, s);
     else if (dtype == CB_F16) launch_dtype<CB_F16>(P, Q, grad_out, grad_w, cls, gc, chunk_bound, num_sms, s);

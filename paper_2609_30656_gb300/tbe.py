@@ -21,6 +21,8 @@ LIB_PATH = os.path.join(_HERE, "libcb_tbe.so")
 CB_OK, CB_ERR_INVALID_ARG, CB_ERR_INDEX_OOB, CB_ERR_BAD_OFFSETS = 0, 1, 2, 3
 CB_ERR_CAPACITY, CB_ERR_OOM, CB_ERR_CUDA, CB_ERR_TIMEOUT = 4, 5, 6, 7
 CB_VALIDATE, CB_TIMING, CB_DEBUG_FORCE_LOOKBACK_TIMEOUT = 0x1, 0x2, 0x100
+CB_OUT_F16, CB_OUT_BF16 = 0x4, 0x8
+_OUT_FLAGS = {torch.float32: 0, torch.float16: CB_OUT_F16, torch.bfloat16: CB_OUT_BF16}
 _DTYPES = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2}
 _POOL = {"sum": 0, "mean": 1}
 _IDX = {torch.int32: 0, torch.int64: 1}
@@ -144,7 +146,8 @@ class TBE:
 
     def __init__(self, tables: list[torch.Tensor], pooling: str = "sum",
                  index_dtype: torch.dtype = torch.int64, validate: bool = False,
-                 timing: bool = False, extra_flags: int = 0):
+                 timing: bool = False, extra_flags: int = 0,
+                 out_dtype: torch.dtype = torch.float32):
         lib = load_library()
         if not tables:
             raise ValueError("at least one table is needed")
@@ -162,10 +165,14 @@ class TBE:
         self.sum_dims = sum(self.dims)
         self.pooling = pooling
         self.index_dtype = index_dtype
+        if out_dtype not in _OUT_FLAGS:
+            raise ValueError(f"unsupported output dtype {out_dtype}")
+        self.out_dtype = out_dtype  # pooled output and grad_out (mixed precision)
         descs = (CbTableDesc * len(tables))(*[
             CbTableDesc(t.data_ptr(), int(t.shape[0]), int(t.shape[1]), _DTYPES[t.dtype])
             for t in tables])
-        flags = (CB_VALIDATE if validate else 0) | (CB_TIMING if timing else 0) | extra_flags
+        flags = ((CB_VALIDATE if validate else 0) | (CB_TIMING if timing else 0) | extra_flags
+                 | _OUT_FLAGS[out_dtype])
         handle = ctypes.c_void_p()
         with torch.cuda.device(self.device):
             _check(lib.cb_tbe_create(descs, len(tables), _POOL[pooling], _IDX[index_dtype], flags,
@@ -211,7 +218,9 @@ class TBE:
         off = self._dev(offsets, self.index_dtype)
         w = self._dev(per_sample_weights, torch.float32)
         if out is None:
-            out = torch.empty(batch, self.sum_dims, dtype=torch.float32, device=self.device)
+            out = torch.empty(batch, self.sum_dims, dtype=self.out_dtype, device=self.device)
+        elif out.dtype != self.out_dtype:
+            raise TypeError(f"out must be {self.out_dtype}")
         with torch.cuda.device(self.device):
             _check(self._lib.cb_tbe_forward(self._h, batch, _ptr(ind), ind.numel(), _ptr(off),
                                             _ptr(w), _ptr(out), self._stream()), "cb_tbe_forward")
@@ -237,7 +246,7 @@ class TBE:
         ind = self._dev(indices, self.index_dtype)
         off = self._dev(offsets, self.index_dtype)
         w = self._dev(per_sample_weights, torch.float32)
-        go = self._dev(grad_out, torch.float32)
+        go = self._dev(grad_out, self.out_dtype)
         cs = CbSparseGrad(
             g.unique_ids.data_ptr(), g.table_offsets.data_ptr(), g.grad_offsets.data_ptr(),
             None if g.grads is None else g.grads.data_ptr(),
@@ -272,7 +281,7 @@ class TBE:
         ind = self._dev(indices, self.index_dtype)
         off = self._dev(offsets, self.index_dtype)
         w = self._dev(per_sample_weights, torch.float32)
-        go = self._dev(grad_out, torch.float32)
+        go = self._dev(grad_out, self.out_dtype)
         ptrs = None
         if optimizer == "adagrad":
             if state is None or len(state) != T:
@@ -297,7 +306,7 @@ class TBE:
         batch = (offsets.numel() - 1) // T
         ind = self._dev(indices, self.index_dtype)
         off = self._dev(offsets, self.index_dtype)
-        go = self._dev(grad_out, torch.float32)
+        go = self._dev(grad_out, self.out_dtype)
         if out is None:
             out = torch.empty(ind.numel(), dtype=torch.float32, device=self.device)
         with torch.cuda.device(self.device):
