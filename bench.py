@@ -224,6 +224,8 @@ def workload_of(args) -> wl.Workload:
     w = wl.get_workload(args.workload)
     if args.tables is not None and args.tables < w.num_tables:
         w = wl.scaled(w, num_tables=args.tables, name=f"{w.name}-first{args.tables}")
+    if getattr(args, "rows", None):
+        w = wl.scaled(w, rows=args.rows, name=f"{w.name}-rows{args.rows}")
     return w
 
 
@@ -781,6 +783,8 @@ def main(argv=None):
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--tables", type=int, default=None,
                     help="first N tables only (a smaller case of the same workload)")
+    ap.add_argument("--rows", type=int, default=None,
+                    help="cap every table's rows (a smaller case for profiling; same lengths and batch)")
     ap.add_argument("--rotate", type=int, default=4)
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-tables", type=int, default=32)
