@@ -403,7 +403,7 @@ def run_ours(args):
                                                               uniq_tables[0], flush, peak)
         # last: it writes the tables
         nxt["backward_apply"] = run_backward_apply(m, w, batches[0], grads_out[0], counts[0],
-                                                   uniq_tables[0], flush, peak, dev)
+                                                   uniq_tables[0], flush, peak, dev, g)
         line["next_rows"] = nxt
     # Component report (Component Benchmark's result table) of this run.
     if args.report and rank == 0:
@@ -567,34 +567,48 @@ def run_mixed_precision(w, tables, b, go, c, uniq, flush, peak):
     return res
 
 
-def run_backward_apply(m, w, b, go, c, uniq, flush, peak, dev):
-    """Backward with SGD / row-wise Adagrad fused (cb_tbe_backward_apply) on one batch.
-    It updates the bench's synthetic tables in place, so it runs after every other
+def run_backward_apply(m, w, b, go, c, uniq, flush, peak, dev, g):
+    """The optimizer step (SGD / row-wise Adagrad) on one batch, fused into the
+    backward (cb_tbe_backward_apply), and as a second pass over the gradient the
+    backward wrote into `g` (cb_tbe_backward + cb_tbe_apply_sparse). It updates
+    the bench's synthetic tables in place, so it runs after every other
     measurement."""
     state = [torch.zeros(r, dtype=torch.float32, device=dev) for r in w.rows]
     res = {}
-    for kind in ("sgd", "adagrad"):
-        def call():
-            m.backward_apply(b.indices, b.offsets, go, b.weights, optimizer=kind, lr=1e-3,
-                             eps=1e-8, state=state if kind == "adagrad" else None)
+    reps = 5
+
+    def timed(calls):
         for _ in range(2):
-            call()
+            for f in calls:
+                f()
         torch.cuda.synchronize()
-        reps = 5
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(reps)]
-        for a, e in ev:
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(calls) + 1)] for _ in range(reps)]
+        for marks in ev:
             flush.zero_()
-            a.record()
-            call()
-            e.record()
+            marks[0].record()
+            for f, e in zip(calls, marks[1:]):
+                f()
+                e.record()
         torch.cuda.synchronize()
         if m.get_error() != 0:
-            raise RuntimeError("device-side error in the fused optimizer step")
-        ms = statistics.mean(a.elapsed_time(e) for a, e in ev)
+            raise RuntimeError("device-side error in the optimizer step")
+        return [statistics.mean(mk[0].elapsed_time(mk[i + 1]) for mk in ev) for i in range(len(calls))]
+
+    for kind in ("sgd", "adagrad"):
+        st = state if kind == "adagrad" else None
+        (ms,) = timed([lambda: m.backward_apply(b.indices, b.offsets, go, b.weights, optimizer=kind, lr=1e-3,
+                                                eps=1e-8, state=st)])
         nbytes = metrics.apply_step_bytes(c, uniq, kind == "adagrad")
         res[kind] = {"ms": round(ms, 4), "alg_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
                      "frac": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4), "bytes": nbytes}
+        bwd_ms, total_ms = timed([lambda: m.backward_into(g, b.indices, b.offsets, go, b.weights),
+                                  lambda: m.apply_sparse(g, optimizer=kind, lr=1e-3, eps=1e-8, state=st)])
+        ab = metrics.sparse_apply_bytes(c, uniq, kind == "adagrad")
+        apply_ms = total_ms - bwd_ms
+        res[f"{kind}_two_pass"] = {"ms": round(total_ms, 4), "backward_ms": round(bwd_ms, 4),
+                                   "apply_ms": round(apply_ms, 4), "apply_bytes": ab,
+                                   "apply_gbs": round(ab / (apply_ms * 1e-3) / 1e9, 1),
+                                   "apply_frac": round(ab / (apply_ms * 1e-3) / 1e9 / peak, 4)}
     del state
     return res
 

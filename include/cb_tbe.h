@@ -213,6 +213,27 @@ cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, i
                                 const void* grad_out, cb_optimizer kind, float lr, float eps,
                                 float* const* state, cudaStream_t stream);
 
+/* The same optimizer step as cb_tbe_backward_apply, applied in a second pass
+ * to a row-sparse gradient that cb_tbe_backward (on this handle) has written:
+ * every row of g->unique_ids[0, U) gets
+ *   CB_OPT_SGD:             E[r] <- E[r] - lr * G
+ *   CB_OPT_ROWWISE_ADAGRAD: m[r] <- m[r] + mean_j G[j]^2;
+ *                           E[r] <- E[r] - lr * G / (sqrt(m[r]) + eps)
+ * in fp32, rounded once to the storage type (round to nearest even). The
+ * result is bit for bit that of cb_tbe_backward_apply on the same batch; this
+ * form keeps the gradient in memory (for clipping, logging or an exchange
+ * between the two passes) and overlaps the rows' loads, where the fused form
+ * writes no gradient buffer.
+ *   g      the buffers of a completed cb_tbe_backward (grads not NULL, 16-byte
+ *          aligned); U and F are read on the device. When that call ran out of
+ *          capacity (U > cap_rows or F > cap_floats) nothing is written.
+ *   kind, lr, eps, state: as in cb_tbe_backward_apply
+ * THIS CALL WRITES THE TABLES given to cb_tbe_create (and the state arrays).
+ * Errors: CB_ERR_INVALID_ARG for a NULL or misaligned buffer, an unknown kind,
+ * a NaN lr, eps < 0 or a missing state; CB_ERR_CUDA if the launch fails. */
+cb_status cb_tbe_apply_sparse(cb_tbe* h, const cb_sparse_grad* g, cb_optimizer kind, float lr, float eps,
+                              float* const* state, cudaStream_t stream);
+
 /* Gradient with respect to the per-sample weights (not in the paper; the
  * pooled bag above is linear in each weight, so this is its exact derivative):
  *   grad_weights[i] = s_b * sum_j grad_out[b, Doff_t + j] * E_t[indices[i], j]

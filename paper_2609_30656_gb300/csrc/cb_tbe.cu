@@ -269,6 +269,11 @@ cb_status check_common(const cb_tbe* h, int32_t batch, const void* indices, int6
     return CB_OK;
 }
 
+bool optimizer_ok(cb_optimizer kind, float lr, float eps, float* const* state) {
+    if (kind != CB_OPT_SGD && kind != CB_OPT_ROWWISE_ADAGRAD) return false;
+    return lr == lr && eps >= 0.f && (kind == CB_OPT_SGD || state);
+}
+
 struct ApplyArgs {
     int kind;
     float lr;
@@ -719,9 +724,7 @@ cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, i
                                 const void* offsets, const float* per_sample_weights,
                                 const void* grad_out, cb_optimizer kind, float lr, float eps,
                                 float* const* state, cudaStream_t stream) {
-    if (!h) return CB_ERR_INVALID_ARG;
-    if (kind != CB_OPT_SGD && kind != CB_OPT_ROWWISE_ADAGRAD) return CB_ERR_INVALID_ARG;
-    if (!(lr == lr) || !(eps >= 0.f) || (kind == CB_OPT_ROWWISE_ADAGRAD && !state)) return CB_ERR_INVALID_ARG;
+    if (!h || !optimizer_ok(kind, lr, eps, state)) return CB_ERR_INVALID_ARG;
     ApplyArgs a;
     a.kind = kind == CB_OPT_SGD ? kApplySgd : kApplyAdagrad;
     a.lr = lr;
@@ -729,6 +732,33 @@ cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, i
     a.state = state;
     return backward_impl(h, batch, indices, num_indices, offsets, per_sample_weights, grad_out, nullptr, &a,
                          stream);
+}
+
+cb_status cb_tbe_apply_sparse(cb_tbe* h, const cb_sparse_grad* g, cb_optimizer kind, float lr, float eps,
+                              float* const* state, cudaStream_t stream) {
+    if (!h || !optimizer_ok(kind, lr, eps, state)) return CB_ERR_INVALID_ARG;
+    if (!g || !g->unique_ids || !g->table_offsets || !g->grad_offsets || !g->grads || !g->num_unique ||
+        !g->num_floats || g->cap_rows < 0 || g->cap_floats < 0 || (reinterpret_cast<uintptr_t>(g->grads) & 15u))
+        return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    h->last_stream = stream;
+    const Problem P = make_problem(h, 0, nullptr, 0, nullptr, nullptr);
+    BwdOut O{};
+    O.unique_ids = g->unique_ids;
+    O.table_offsets = g->table_offsets;
+    O.grad_offsets = g->grad_offsets;
+    O.grads = g->grads;
+    O.cap_rows = g->cap_rows;
+    O.cap_floats = g->cap_floats;
+    O.num_unique = g->num_unique;
+    O.num_floats = g->num_floats;
+    O.apply = kind == CB_OPT_SGD ? kApplySgd : kApplyAdagrad;
+    O.lr = lr;
+    O.eps = eps;
+    O.state = state;
+    launch_apply_sparse(P, O, h->num_sms, stream);
+    h->launches += 1;
+    return finish_call(h, stream);
 }
 
 cb_status cb_tbe_get_error(cb_tbe* h) {

@@ -307,7 +307,7 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_apply_split_kernel(const __g
             float sq = 0.f;
             for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
                 const float4 v = *reinterpret_cast<const float4*>(g + x0);
-                sq += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+                sq += sq4(v);
             }
             const float scale = step_scale(O, t, row, td.dim, sq);
             for (int x0 = lane * 4; x0 < td.dim; x0 += 128)
@@ -373,6 +373,125 @@ void launch_bwd_apply_split(const Problem& P, const Plan& Q, const BwdOut& O, in
     const int64_t need = (chunk_bound + kWarpThreads - 1) / kWarpThreads;  // 32 chunks per warp
     const int grid = static_cast<int>(max64(1, min64(need, static_cast<int64_t>(num_sms) * 8)));
     bwd_apply_split_kernel<<<grid, kWarpThreads, 0, s>>>(P, Q, O);
+}
+
+}  // namespace cbtbe
+
+namespace cbtbe {
+
+// ---------------------------------------------------------------- (7) sparse step
+
+// The optimizer step from a row-sparse gradient already in memory (written by
+// the backward). Every touched row is independent: a warp takes 32 rows, each
+// lane fetches one row's id and gradient offset and finds its table by
+// bisection over the per-table ranges (one round trip for all 32), then the
+// warp steps the rows R at a time, issuing all their gradient, table and state
+// loads before any store. Lane l owns columns 4l + 128m, m < M (the fused
+// step's order, so both give the same sums of squares). Nothing is done when
+// the gradient buffers were too small (the backward then wrote no rows).
+template <int M, int R>
+__global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid_constant__ Problem P,
+                                                                    const __grid_constant__ BwdOut O) {
+    static_assert(32 % R == 0, "rows per step divide the warp's 32");
+    const int lane = threadIdx.x & 31;
+    const int64_t U = *O.num_unique;
+    if (U > O.cap_rows || *O.num_floats > O.cap_floats) return;
+    const bool adagrad = O.apply == kApplyAdagrad;
+    for (int64_t u0 = warp_id_global() * 32; u0 < U; u0 += warps_in_grid() * 32) {
+        // this lane's row: start of its stored row, of its gradient and state
+        const int64_t u = min64(u0 + lane, U - 1);
+        const int64_t id = __ldg(O.unique_ids + u);
+        const int64_t goff = __ldg(O.grad_offsets + u);
+        int lo = 0, hi = P.T;  // table_offsets[lo] <= u < table_offsets[lo + 1]
+        while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (__ldg(O.table_offsets + mid) <= u) lo = mid;
+            else hi = mid;
+        }
+        const TableDev& td = P.tables[lo];
+        const int64_t row = id - td.row_base;
+        const unsigned long long my_row = reinterpret_cast<unsigned long long>(row_ptr(td, row));
+        const unsigned long long my_grad = reinterpret_cast<unsigned long long>(O.grads + goff);
+        const unsigned long long my_state =
+            adagrad ? reinterpret_cast<unsigned long long>(O.state[lo] + row) : 0ull;
+        const int my_shape = (td.dim << 2) | td.dtype;
+        const float my_m0 = adagrad ? *reinterpret_cast<const float*>(my_state) : 0.f;
+        const int rows_here = static_cast<int>(min64(32, U - u0));
+        for (int r0 = 0; r0 < rows_here; r0 += R) {
+            char* rp[R];
+            int shape[R];
+            float4 g[R][M];
+            uint4 x[R][M];
+#pragma unroll
+            for (int i = 0; i < R; ++i) {
+                rp[i] = reinterpret_cast<char*>(__shfl_sync(kFull, my_row, r0 + i));
+                const float* gp = reinterpret_cast<const float*>(__shfl_sync(kFull, my_grad, r0 + i));
+                shape[i] = __shfl_sync(kFull, my_shape, r0 + i);
+#pragma unroll
+                for (int m = 0; m < M; ++m) {
+                    const int x0 = lane * 4 + 128 * m;
+                    if (x0 < (shape[i] >> 2)) {
+                        g[i][m] = *reinterpret_cast<const float4*>(gp + x0);
+                        x[i][m] = load_cols(rp[i], shape[i] & 3, x0);
+                    }
+                }
+            }
+            float scale[R];
+#pragma unroll
+            for (int i = 0; i < R; ++i) scale[i] = O.lr;
+            if (adagrad) {
+                // The Adagrad scale with the arithmetic of adagrad_scale: the R
+                // rows' butterflies interleaved, then lane r0 + i, which holds
+                // row r0 + i's state, takes that row's update.
+                float sq[R];
+#pragma unroll
+                for (int i = 0; i < R; ++i) {
+                    sq[i] = 0.f;
+#pragma unroll
+                    for (int m = 0; m < M; ++m)
+                        if (lane * 4 + 128 * m < (shape[i] >> 2)) sq[i] += sq4(g[i][m]);
+                }
+#pragma unroll
+                for (int off = 16; off >= 1; off >>= 1)
+#pragma unroll
+                    for (int i = 0; i < R; ++i) sq[i] += __shfl_xor_sync(kFull, sq[i], off);
+                float mine = 0.f;
+#pragma unroll
+                for (int i = 0; i < R; ++i)
+                    if (lane == r0 + i) mine = sq[i];
+                float my_scale = O.lr;
+                if (lane >= r0 && lane < r0 + R && lane < rows_here) {
+                    const float m = my_m0 + mine / static_cast<float>(my_shape >> 2);
+                    *reinterpret_cast<float*>(my_state) = m;
+                    my_scale = O.lr / (sqrtf(m) + O.eps);
+                }
+#pragma unroll
+                for (int i = 0; i < R; ++i) scale[i] = __shfl_sync(kFull, my_scale, r0 + i);
+            }
+#pragma unroll
+            for (int i = 0; i < R; ++i) {
+                if (r0 + i >= rows_here) break;  // warp-uniform
+                const int dim = shape[i] >> 2;
+#pragma unroll
+                for (int m = 0; m < M; ++m) {
+                    const int x0 = lane * 4 + 128 * m;
+                    if (x0 < dim) store_step(rp[i], shape[i] & 3, x0, x[i][m], g[i][m], scale[i]);
+                }
+            }
+        }
+    }
+}
+
+template <int M, int R>
+void launch_apply_sparse_m(const Problem& P, const BwdOut& O, int num_sms, cudaStream_t s) {
+    static int cap = occupancy_grid(apply_sparse_kernel<M, R>, kWarpThreads, num_sms);
+    apply_sparse_kernel<M, R><<<cap, kWarpThreads, 0, s>>>(P, O);
+}
+
+void launch_apply_sparse(const Problem& P, const BwdOut& O, int num_sms, cudaStream_t s) {
+    if (P.dmax <= 128) launch_apply_sparse_m<1, 8>(P, O, num_sms, s);
+    else if (P.dmax <= 256) launch_apply_sparse_m<2, 4>(P, O, num_sms, s);
+    else launch_apply_sparse_m<4, 2>(P, O, num_sms, s);
 }
 
 }  // namespace cbtbe

@@ -71,6 +71,8 @@ constexpr int kApplySgd = 1;
 constexpr int kApplyAdagrad = 2;
 
 void launch_validate_offsets(const Problem& P, int num_sms, cudaStream_t s);
+// The optimizer step of O.apply from the row-sparse gradient in O's caller buffers.
+void launch_apply_sparse(const Problem& P, const BwdOut& O, int num_sms, cudaStream_t s);
 void launch_plan(const Problem& P, const Plan& Q, int mode, const uint32_t* seg_start,
                  const int64_t* num_unique, int num_sms, bool tables_too, cudaStream_t s);
 

@@ -32,41 +32,74 @@ inline int warp_grid(int64_t chunk_bound, int cap) {
 
 // ---------------------------------------------------------------- optimizer step
 
-// new = E - scale * g for four consecutive columns of a stored row, rounded
-// once from fp32 to the storage type (round to nearest even).
-__device__ __forceinline__ void step_cols(const TableDev& td, int64_t row, int col, float4 g, float scale) {
-    const int64_t k = row * td.dim + col;
-    if (td.dtype == CB_F32) {
-        float4* p = reinterpret_cast<float4*>(const_cast<void*>(td.data)) + k / 4;
-        float4 x = *p;
-        x.x = fmaf(-scale, g.x, x.x);
-        x.y = fmaf(-scale, g.y, x.y);
-        x.z = fmaf(-scale, g.z, x.z);
-        x.w = fmaf(-scale, g.w, x.w);
-        *p = x;
-    } else if (td.dtype == CB_F16) {
-        uint2* p = reinterpret_cast<uint2*>(const_cast<void*>(td.data)) + k / 4;
-        uint2 x = *p;
+// Start of a stored row.
+__device__ __forceinline__ char* row_ptr(const TableDev& td, int64_t row) {
+    return static_cast<char*>(const_cast<void*>(td.data)) + row * td.dim * dtype_bytes(td.dtype);
+}
+
+// The stored bits of four consecutive columns of a row: 16 bytes (fp32) or
+// 8 bytes in .x, .y (fp16 / bf16).
+__device__ __forceinline__ uint4 load_cols(const char* rowp, int dtype, int col) {
+    if (dtype == CB_F32) return *reinterpret_cast<const uint4*>(rowp + 4 * col);
+    const uint2 x = *reinterpret_cast<const uint2*>(rowp + 2 * col);
+    return make_uint4(x.x, x.y, 0u, 0u);
+}
+
+// new = E - scale * g for the four columns whose stored bits are `x`, rounded
+// once from fp32 to the storage type (round to nearest even), and stored.
+__device__ __forceinline__ void store_step(char* rowp, int dtype, int col, uint4 x, float4 g, float scale) {
+    if (dtype == CB_F32) {
+        float4 v = make_float4(__uint_as_float(x.x), __uint_as_float(x.y), __uint_as_float(x.z),
+                               __uint_as_float(x.w));
+        v.x = fmaf(-scale, g.x, v.x);
+        v.y = fmaf(-scale, g.y, v.y);
+        v.z = fmaf(-scale, g.z, v.z);
+        v.w = fmaf(-scale, g.w, v.w);
+        *reinterpret_cast<float4*>(rowp + 4 * col) = v;
+        return;
+    }
+    uint2 y;
+    if (dtype == CB_F16) {
         __half2 a, b;
         memcpy(&a, &x.x, 4);
         memcpy(&b, &x.y, 4);
         const float2 fa = __half22float2(a), fb = __half22float2(b);
         a = __floats2half2_rn(fmaf(-scale, g.x, fa.x), fmaf(-scale, g.y, fa.y));
         b = __floats2half2_rn(fmaf(-scale, g.z, fb.x), fmaf(-scale, g.w, fb.y));
-        memcpy(&x.x, &a, 4);
-        memcpy(&x.y, &b, 4);
-        *p = x;
+        memcpy(&y.x, &a, 4);
+        memcpy(&y.y, &b, 4);
     } else {
-        uint2* p = reinterpret_cast<uint2*>(const_cast<void*>(td.data)) + k / 4;
-        uint2 x = *p;
         const float f0 = __uint_as_float(x.x << 16), f1 = __uint_as_float(x.x & 0xffff0000u);
         const float f2 = __uint_as_float(x.y << 16), f3 = __uint_as_float(x.y & 0xffff0000u);
         const __nv_bfloat162 a = __floats2bfloat162_rn(fmaf(-scale, g.x, f0), fmaf(-scale, g.y, f1));
         const __nv_bfloat162 b = __floats2bfloat162_rn(fmaf(-scale, g.z, f2), fmaf(-scale, g.w, f3));
-        memcpy(&x.x, &a, 4);
-        memcpy(&x.y, &b, 4);
-        *p = x;
+        memcpy(&y.x, &a, 4);
+        memcpy(&y.y, &b, 4);
     }
+    *reinterpret_cast<uint2*>(rowp + 2 * col) = y;
+}
+
+__device__ __forceinline__ void step_cols(const TableDev& td, int64_t row, int col, float4 g, float scale) {
+    char* p = row_ptr(td, row);
+    store_step(p, td.dtype, col, load_cols(p, td.dtype, col), g, scale);
+}
+
+// This lane's share of sum g^2 over four columns (the same expression in the
+// fused and the two-pass step, so both give the same Adagrad state).
+__device__ __forceinline__ float sq4(float4 g) { return g.x * g.x + g.y * g.y + g.z * g.z + g.w * g.w; }
+
+// The Adagrad scale from the summed squares and the row's previous state `m0`
+// (meaningful in lane 0); lane 0 stores the new state.
+__device__ __forceinline__ float adagrad_scale(const BwdOut& O, float* st, int dim, float sq, float m0) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) sq += __shfl_xor_sync(kFull, sq, off);
+    float m = 0.f;
+    if ((threadIdx.x & 31) == 0) {
+        m = m0 + sq / static_cast<float>(dim);
+        *st = m;
+    }
+    m = __shfl_sync(kFull, m, 0);
+    return O.lr / (sqrtf(m) + O.eps);
 }
 
 // The step's scale for one row: lr (SGD), or lr / (sqrt(m) + eps) after
@@ -74,16 +107,8 @@ __device__ __forceinline__ void step_cols(const TableDev& td, int64_t row, int c
 // share of sum g^2; the whole warp calls this, lane 0 owns the state word.
 __device__ __forceinline__ float step_scale(const BwdOut& O, int t, int64_t row, int dim, float sq) {
     if (O.apply != kApplyAdagrad) return O.lr;
-#pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) sq += __shfl_xor_sync(kFull, sq, off);
-    float m = 0.f;
-    if ((threadIdx.x & 31) == 0) {
-        float* st = O.state[t] + row;
-        m = *st + sq / static_cast<float>(dim);
-        *st = m;
-    }
-    m = __shfl_sync(kFull, m, 0);
-    return O.lr / (sqrtf(m) + O.eps);
+    float* st = O.state[t] + row;
+    return adagrad_scale(O, st, dim, sq, (threadIdx.x & 31) == 0 ? *st : 0.f);
 }
 
 // The fused step on one complete run's row, as the walker holds it: lane v of
@@ -106,7 +131,7 @@ __device__ __noinline__ void apply_row(const Problem& P, const BwdOut& O, int t,
 #pragma unroll
     for (int k = 0; k < N; ++k)
         if (group0 && g.col[k] >= 0)
-            sq += g.v[k].x * g.v[k].x + g.v[k].y * g.v[k].y + g.v[k].z * g.v[k].z + g.v[k].w * g.v[k].w;
+            sq += sq4(g.v[k]);
     const float scale = step_scale(O, t, row, td.dim, sq);
     if (!group0) return;
 #pragma unroll

@@ -106,6 +106,17 @@ def apply_step_bytes(c: BatchCounts, unique_per_table, adagrad: bool) -> int:
     return (b["total"] - b["grads"] - b["unique_ids"] + 2 * rows + (8 * U if adagrad else 0))
 
 
+def sparse_apply_bytes(c: BatchCounts, unique_per_table, adagrad: bool) -> int:
+    """Algorithmic bytes of the optimizer step as a second pass over a written
+    row-sparse gradient: per touched row its id and offset (8 + 8 bytes), its
+    fp32 gradient row, the table row read and written in its storage type, and
+    for row-wise Adagrad its fp32 state word read and written."""
+    U = int(sum(int(u) for u in unique_per_table))
+    grads = sum(int(u) * d * 4 for u, d in zip(unique_per_table, c.dims))
+    rows = sum(int(u) * d * c.elem_bytes for u, d in zip(unique_per_table, c.dims))
+    return 16 * U + grads + 2 * rows + (8 * U if adagrad else 0)
+
+
 def sort_bytes(n: int, passes: int) -> int:
     return 16 * n * passes
 

@@ -32,7 +32,7 @@ EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
            "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad",
-           "cb_tbe_backward_apply", "cb_kjt_replicate")
+           "cb_tbe_backward_apply", "cb_tbe_apply_sparse", "cb_kjt_replicate")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -84,6 +84,8 @@ def load_library() -> ctypes.CDLL:
     lib.cb_tbe_weight_grad.argtypes = [p, i32, p, i64, p, p, p, p]
     lib.cb_tbe_backward_apply.argtypes = [p, i32, p, i64, p, p, p, ctypes.c_int, ctypes.c_float,
                                           ctypes.c_float, p, p]
+    lib.cb_tbe_apply_sparse.argtypes = [p, ctypes.POINTER(CbSparseGrad), ctypes.c_int, ctypes.c_float,
+                                        ctypes.c_float, p, p]
     lib.cb_kjt_replicate.argtypes = [p, p, p, ctypes.c_int, i32, i32, i64, i32, p, p, p, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
@@ -273,31 +275,53 @@ class TBE:
         """Backward with the optimizer step fused (cb_tbe_backward_apply): updates the
         tables this handle was created with (and, for "adagrad", the fp32 [rows_t]
         state tensors) in place."""
-        kinds = {"sgd": 0, "adagrad": 1}
-        if optimizer not in kinds:
-            raise ValueError(f"unknown optimizer {optimizer!r}")
+        kind, ptrs = self._optimizer_args(optimizer, state)
         T = len(self.dims)
         batch = (offsets.numel() - 1) // T
         ind = self._dev(indices, self.index_dtype)
         off = self._dev(offsets, self.index_dtype)
         w = self._dev(per_sample_weights, torch.float32)
         go = self._dev(grad_out, self.out_dtype)
-        ptrs = None
-        if optimizer == "adagrad":
-            if state is None or len(state) != T:
-                raise ValueError("adagrad needs one fp32 state tensor per table")
-            for s_, r in zip(state, self.rows):
-                if (s_.device != self.device or s_.dtype != torch.float32 or s_.numel() != r
-                        or not s_.is_contiguous()):
-                    raise ValueError("state[t] must be a contiguous fp32 [rows_t] tensor on the device")
-            ptrs = torch.tensor([s_.data_ptr() for s_ in state], dtype=torch.int64,
-                                device=self.device)
         with torch.cuda.device(self.device):
             _check(self._lib.cb_tbe_backward_apply(self._h, batch, _ptr(ind), ind.numel(), _ptr(off),
-                                                   _ptr(w), _ptr(go), kinds[optimizer], lr, eps,
+                                                   _ptr(w), _ptr(go), kind, lr, eps,
                                                    _ptr(ptrs), self._stream()),
                    "cb_tbe_backward_apply")
         self._keep = ptrs  # the pointer array must outlive the enqueued work
+
+    def apply_sparse(self, g: SparseGrad, optimizer: str = "sgd", lr: float = 0.01,
+                     eps: float = 1e-8, state: list[torch.Tensor] | None = None) -> None:
+        """The optimizer step of backward_apply from a gradient that backward /
+        backward_into wrote (cb_tbe_apply_sparse): same update, bit for bit."""
+        if g.grads is None:
+            raise ValueError("a size-only gradient holds no values")
+        kind, ptrs = self._optimizer_args(optimizer, state)
+        cs = CbSparseGrad(g.unique_ids.data_ptr(), g.table_offsets.data_ptr(), g.grad_offsets.data_ptr(),
+                          g.grads.data_ptr(), g.unique_ids.numel(), g.grads.numel(),
+                          g.num_unique_dev.data_ptr(), g.num_floats_dev.data_ptr())
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_apply_sparse(self._h, ctypes.byref(cs), kind, lr, eps, _ptr(ptrs),
+                                                 self._stream()), "cb_tbe_apply_sparse")
+        self._keep = ptrs
+
+    def _optimizer_args(self, optimizer: str, state):
+        kinds = {"sgd": 0, "adagrad": 1}
+        if optimizer not in kinds:
+            raise ValueError(f"unknown optimizer {optimizer!r}")
+        if optimizer != "adagrad":
+            return kinds[optimizer], None
+        if state is None or len(state) != len(self.dims):
+            raise ValueError("adagrad needs one fp32 state tensor per table")
+        for s_, r in zip(state, self.rows):
+            if (s_.device != self.device or s_.dtype != torch.float32 or s_.numel() != r
+                    or not s_.is_contiguous()):
+                raise ValueError("state[t] must be a contiguous fp32 [rows_t] tensor on the device")
+        key = tuple(s_.data_ptr() for s_ in state)
+        cached = getattr(self, "_state_ptrs", None)
+        if cached is None or cached[0] != key:  # one small copy per new set of state tensors
+            cached = (key, torch.tensor(key, dtype=torch.int64, device=self.device))
+            self._state_ptrs = cached
+        return kinds[optimizer], cached[1]
 
     def weight_grad(self, indices, offsets, grad_out,
                     out: torch.Tensor | None = None) -> torch.Tensor:

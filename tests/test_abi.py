@@ -79,6 +79,7 @@ def test_host_side_argument_errors_return_before_any_gpu_work(lib):
     assert lib.cb_tbe_weight_grad(None, 1, None, 0, None, None, None, None) == tbe.CB_ERR_INVALID_ARG
     assert lib.cb_tbe_backward_apply(None, 1, None, 0, None, None, None, 0, 0.1, 0.0, None,
                                      None) == tbe.CB_ERR_INVALID_ARG
+    assert lib.cb_tbe_apply_sparse(None, None, 0, 0.1, 0.0, None, None) == tbe.CB_ERR_INVALID_ARG
 
 
 def test_product_path_fails_loudly_without_the_library(monkeypatch, tmp_path):

@@ -45,6 +45,17 @@ def test_apply_step_bytes_by_hand():
     assert metrics.apply_step_bytes(c, [3, 1], True) == metrics.apply_step_bytes(c, [3, 1], False) + 4 * 8
 
 
+def test_sparse_apply_bytes_by_hand():
+    # 3 touched rows of the dim-4 fp16 table, 1 of the dim-8 one
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts((4, 8), 2, 3, off, weighted=False)
+    ids = 4 * 16
+    grads = (3 * 4 + 8) * 4
+    rows = 2 * (3 * 4 + 8) * 2
+    assert metrics.sparse_apply_bytes(c, [3, 1], False) == ids + grads + rows
+    assert metrics.sparse_apply_bytes(c, [3, 1], True) == ids + grads + rows + 4 * 8
+
+
 def test_fm_bytes_by_hand():
     # 3 samples x 2 fields x dim 4: 24 floats of pooled rows
     assert metrics.fm_bytes(3, 2, 4, backward=False) == 24 * 4 + 3 * 4
