@@ -42,14 +42,18 @@ __device__ __forceinline__ void store_volatile(uint32_t* p, uint32_t v) {
 
 constexpr int kLookbackWindow = 8;  // predecessor tiles inspected per look-back round
 
+__device__ __forceinline__ uint32_t sort_digit(uint32_t key, uint32_t row_base, int shift) {
+    return ((key - row_base) >> shift) & (kRadix - 1);
+}
+
 __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     extern __shared__ __align__(16) uint32_t sh_dyn[];
-    uint32_t* sh_keys = sh_dyn;                        // tile-sorted keys
-    uint32_t* sh_vals = sh_dyn + kSortTile;            // tile-sorted payloads
-    uint32_t* sh_vals_in = sh_dyn + 2 * kSortTile;     // payloads in load order
-    __shared__ uint32_t sh_warp[kSortWarps][kRadix];   // per-warp counts, then prefixes
-    __shared__ uint32_t sh_start[kRadix];              // tile-local start of each digit
-    __shared__ long long sh_goff[kRadix];              // global destination - local index
+    uint32_t* sh_keys = sh_dyn;                            // tile-sorted keys
+    uint32_t* sh_vals = sh_dyn + kSortTile;                // tile-sorted payloads
+    __shared__ uint32_t sh_warp[kSortWarps][kRadix + 1];   // per-warp counts, then prefixes
+                                                           // (slot kRadix: positions past the tile)
+    __shared__ uint32_t sh_start[kRadix];                  // tile-local start of each digit
+    __shared__ int32_t sh_goff[kRadix];                    // global destination - local index
     __shared__ int64_t sh_scan[33];
     __shared__ uint32_t sh_tile;
     __shared__ int sh_abort;
@@ -59,7 +63,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         sh_tile = atomicAdd(S.tile_counter, 1u);
         sh_abort = 0;
     }
-    for (int i = tid; i < kSortWarps * kRadix; i += kSortThreads) (&sh_warp[0][0])[i] = 0;
+    for (int i = tid; i < kSortWarps * (kRadix + 1); i += kSortThreads) (&sh_warp[0][0])[i] = 0;
     __syncthreads();
     const uint32_t tile = sh_tile;
     if (tile >= *S.num_tiles) return;  // the grid is an upper bound on the tiles
@@ -71,33 +75,32 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     const int64_t first_tile = S.table_first_tile[t];
 
     // Warp-striped load: item j of lane l is position tile_base + wid*512 + j*32 + l.
-    // Payloads wait in shared memory; keys and ranks stay in registers.
-    uint32_t key[kSortItems];
+    // Keys, payloads and ranks stay in registers until the shared scatter.
+    uint32_t key[kSortItems], val[kSortItems];
+#pragma unroll
+    for (int j = 0; j < kSortItems; ++j) {
+        const int local = wid * (32 * kSortItems) + j * 32 + lane;
+        const bool valid = local < tile_count;
+        key[j] = valid ? __ldg(S.keys_in + tile_base + local) : 0u;
+        val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
+    }
+    // Stable rank within the warp: the lanes holding one digit in item j find
+    // each other (match), their lowest lane adds their number to the warp's
+    // counter of that digit and shares the old value. A warp's shared-memory
+    // atomics take effect in issue order, so item j's lanes count before item
+    // j + 1's, and lanes of one item by lane: the rank follows the position.
+    const uint32_t lt_mask = (1u << lane) - 1u;
     uint32_t rank2[kSortItems / 2];  // two 16-bit ranks per register
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
-        const bool valid = local < tile_count;
-        key[j] = valid ? __ldg(S.keys_in + tile_base + local) : 0xffffffffu;
-        if (valid) sh_vals_in[local] = __ldg(S.vals_in + tile_base + local);
-    }
-    const uint32_t lt_mask = (1u << lane) - 1u;
-#pragma unroll
-    for (int j = 0; j < kSortItems; ++j) {
-        const int local = wid * (32 * kSortItems) + j * 32 + lane;
-        const bool valid = local < tile_count;
-        const uint32_t vmask = __ballot_sync(kFull, valid);
-        const uint32_t d = ((key[j] - row_base) >> S.shift) & (kRadix - 1);
-        uint32_t peers = 0, before = 0, r = 0;
-        if (valid) {
-            peers = __match_any_sync(vmask, d);
-            before = sh_warp[wid][d];
-            r = before + __popc(peers & lt_mask);
-        }
+        const uint32_t d = local < tile_count ? sort_digit(key[j], row_base, S.shift) : kRadix;
+        const uint32_t peers = __match_any_sync(kFull, d);
+        const int leader = __ffs(peers) - 1;
+        uint32_t before = 0;
+        if (lane == leader) before = atomicAdd(&sh_warp[wid][d], static_cast<uint32_t>(__popc(peers)));
+        const uint32_t r = __shfl_sync(kFull, before, leader) + __popc(peers & lt_mask);
         if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;
-        __syncwarp();
-        if (valid && lane == __ffs(peers) - 1) sh_warp[wid][d] = before + __popc(peers);
-        __syncwarp();
     }
     __syncthreads();
 
@@ -168,31 +171,54 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         }
         store_volatile(my_status, kFlagIncl | ((excl + count) & kCountMask));
     }
-    sh_goff[d] = static_cast<long long>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) +
-                 excl - static_cast<long long>(start);
+    // Positions are below 2^30 and the local index below 2^12: 32 bits suffice.
+    sh_goff[d] = static_cast<int32_t>(
+        static_cast<int64_t>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) + excl - start);
     __syncthreads();
 
-    // Scatter into shared memory in tile-sorted order.
+    // Scatter into shared memory in tile-sorted order: every slot first (the
+    // counters are read-only here), then the stores.
+#pragma unroll
+    for (int j = 0; j < kSortItems; ++j) {
+        const uint32_t dd = sort_digit(key[j], row_base, S.shift);
+        const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
+        const uint32_t pos = (sh_start[dd] + sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
+        rank2[j >> 1] = (j & 1) ? ((rank2[j >> 1] & 0xffffu) | (pos << 16))
+                                : ((rank2[j >> 1] & 0xffff0000u) | pos);
+    }
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         if (local < tile_count) {
-            const uint32_t dd = ((key[j] - row_base) >> S.shift) & (kRadix - 1);
-            const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
-            const uint32_t pos = sh_start[dd] + sh_warp[wid][dd] + r;
+            const uint32_t pos = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
             sh_keys[pos] = key[j];
-            sh_vals[pos] = sh_vals_in[local];
+            sh_vals[pos] = val[j];
         }
     }
     __syncthreads();
     if (sh_abort) return;
     // Consecutive shared slots of one digit go to consecutive global slots.
-    for (int i = tid; i < tile_count; i += kSortThreads) {
-        const uint32_t k2 = sh_keys[i];
-        const long long dest = sh_goff[((k2 - row_base) >> S.shift) & (kRadix - 1)] + i;
-        if (dest >= 0 && dest < S.n) {
-            S.keys_out[dest] = k2;
-            S.vals_out[dest] = sh_vals[i];
+    // Half a tile at a time: its shared reads, its destinations, its stores.
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        constexpr int kHalf = kSortItems / 2;
+        int32_t dst[kHalf];
+#pragma unroll
+        for (int j = 0; j < kHalf; ++j) {
+            const int i = tid + (h * kHalf + j) * kSortThreads;
+            key[j] = i < tile_count ? sh_keys[i] : 0u;
+            val[j] = i < tile_count ? sh_vals[i] : 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < kHalf; ++j)
+            dst[j] = sh_goff[sort_digit(key[j], row_base, S.shift)] + tid + (h * kHalf + j) * kSortThreads;
+#pragma unroll
+        for (int j = 0; j < kHalf; ++j) {
+            const int i = tid + (h * kHalf + j) * kSortThreads;
+            if (i < tile_count && dst[j] >= 0 && dst[j] < S.n) {
+                S.keys_out[dst[j]] = key[j];
+                S.vals_out[dst[j]] = val[j];
+            }
         }
     }
 }
@@ -271,7 +297,7 @@ void launch_sort_bases(const uint32_t* hist, const int64_t* table_pos, int T, in
     sort_base_kernel<<<T, kRadix, 0, s>>>(hist, table_pos, passes, base);
 }
 
-constexpr int kSortDynSmem = 3 * kSortTile * sizeof(uint32_t);  // 48 KB
+constexpr int kSortDynSmem = 2 * kSortTile * sizeof(uint32_t);  // 32 KB
 
 void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     static bool configured = false;
