@@ -71,8 +71,15 @@ typedef enum { CB_I32 = 0, CB_I64 = 1 } cb_index_dtype;
  * the two; every table's dim must then be a multiple of 8. Default: fp32. */
 #define CB_OUT_F16  0x4u
 #define CB_OUT_BF16 0x8u
-/* Test hook: the first radix pass's tile 1 waits on a status word that nothing
- * writes, so its bounded wait runs out and the call reports CB_ERR_TIMEOUT. */
+/* The backward's radix passes as single sweeps with a decoupled look-back
+ * (each pair read and written once per pass; a block waits, bounded in time,
+ * for the counts its table's earlier tiles publish) instead of the default
+ * reduce-then-scan passes (a counting read of the keys and a scan of the tile
+ * counts before each scatter; no block waits on another). Same results. */
+#define CB_SORT_LOOKBACK 0x200u
+/* Test hook (implies CB_SORT_LOOKBACK): the first radix pass's tile 1 waits on
+ * a status word that nothing writes, so its bounded wait runs out and the call
+ * reports CB_ERR_TIMEOUT. */
 #define CB_DEBUG_FORCE_LOOKBACK_TIMEOUT 0x100u
 
 /* One embedding table: `rows` x `dim` values of `dtype`, row-major, at the

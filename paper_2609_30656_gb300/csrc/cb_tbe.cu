@@ -73,6 +73,9 @@ struct Workspace {
     uint32_t* digit_base = nullptr;
     uint32_t* status = nullptr;
     uint32_t* tile_counters = nullptr;
+    uint32_t* tile_digits = nullptr;
+    uint32_t* seg_sums = nullptr;
+    int segments = 1;
     int64_t* tile_heads = nullptr;
     int64_t* tile_base = nullptr;
     uint32_t* uniq = nullptr;
@@ -163,15 +166,21 @@ size_t layout(const cb_tbe* h, int64_t B, int64_t n, char* base, Workspace* w) {
     ws.sp_class_base = static_cast<int64_t*>(take(sizeof(int64_t) * 2));
     ws.sp_tiles = static_cast<Chunk*>(take(sizeof(Chunk) * ws.sp_max_tiles));
     ws.sort_tiles = ws.sp_max_tiles;
-    const size_t hist_words = static_cast<size_t>(T) * h->passes * 256;
-    ws.digit_base = static_cast<uint32_t*>(take(sizeof(uint32_t) * hist_words));
-    ws.status_bytes = sizeof(uint32_t) * static_cast<size_t>(h->passes) * ws.sort_tiles * 256;
-    // histograms, status words and tile counters are adjacent: one memset clears them
-    ws.hist = static_cast<uint32_t*>(take(sizeof(uint32_t) * hist_words + ws.status_bytes +
-                                          sizeof(uint32_t) * 4));
-    ws.status = base ? ws.hist + hist_words : nullptr;
-    ws.tile_counters = base ? ws.status + static_cast<size_t>(h->passes) * ws.sort_tiles * 256 : nullptr;
-    ws.status_bytes += sizeof(uint32_t) * hist_words;  // bytes cleared from `hist` on
+    if (h->flags & (CB_SORT_LOOKBACK | CB_DEBUG_FORCE_LOOKBACK_TIMEOUT)) {
+        const size_t hist_words = static_cast<size_t>(T) * h->passes * 256;
+        ws.digit_base = static_cast<uint32_t*>(take(sizeof(uint32_t) * hist_words));
+        ws.status_bytes = sizeof(uint32_t) * static_cast<size_t>(h->passes) * ws.sort_tiles * 256;
+        // histograms, status words and tile counters are adjacent: one memset clears them
+        ws.hist = static_cast<uint32_t*>(take(sizeof(uint32_t) * hist_words + ws.status_bytes +
+                                              sizeof(uint32_t) * 4));
+        ws.status = base ? ws.hist + hist_words : nullptr;
+        ws.tile_counters = base ? ws.status + static_cast<size_t>(h->passes) * ws.sort_tiles * 256 : nullptr;
+        ws.status_bytes += sizeof(uint32_t) * hist_words + sizeof(uint32_t) * 4;  // cleared from `hist` on
+    } else {
+        ws.segments = radix_segments(ws.sp_max_tiles, static_cast<int>(T));
+        ws.tile_digits = static_cast<uint32_t*>(take(sizeof(uint32_t) * 256 * ws.sort_tiles));
+        ws.seg_sums = static_cast<uint32_t*>(take(sizeof(uint32_t) * 256 * T * ws.segments));
+    }
     const int64_t rt = rle_num_tiles(n);
     ws.tile_heads = static_cast<int64_t*>(take(sizeof(int64_t) * rt));
     ws.tile_base = static_cast<int64_t*>(take(sizeof(int64_t) * rt));
@@ -321,8 +330,8 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     // (1) keys and payloads
     launch_plan(P, Q, 0, nullptr, nullptr, h->num_sms, true, stream);
     h->launches += 2;
-    if (cudaMemsetAsync(w.hist, 0, w.status_bytes + sizeof(uint32_t) * 4, stream) != cudaSuccess)
-        return CB_ERR_CUDA;
+    const bool lookback = (h->flags & (CB_SORT_LOOKBACK | CB_DEBUG_FORCE_LOOKBACK_TIMEOUT)) != 0;
+    if (lookback && cudaMemsetAsync(w.hist, 0, w.status_bytes, stream) != cudaSuccess) return CB_ERR_CUDA;
     KeyGen K;
     K.keys = w.keys[0];
     K.vals = w.vals[0];
@@ -346,13 +355,16 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     SQ.carry_head = SQ.carry_tail = nullptr;
     SQ.tail_owner = nullptr;
     launch_plan(P, SQ, 2, nullptr, nullptr, h->num_sms, true, stream);
-    launch_sort_hist(w.keys[0], w.sp_tiles, w.sp_class_base + 1, w.sp_max_tiles, h->d_tables,
-                     h->passes, w.hist, h->num_sms, stream);
-    launch_sort_bases(w.hist, w.sp_table_pos, h->T, h->passes, w.digit_base, stream);
-    h->launches += 4;
+    h->launches += 2;
+    if (lookback) {
+        launch_sort_hist(w.keys[0], w.sp_tiles, w.sp_class_base + 1, w.sp_max_tiles, h->d_tables,
+                         h->passes, w.hist, h->num_sms, stream);
+        launch_sort_bases(w.hist, w.sp_table_pos, h->T, h->passes, w.digit_base, stream);
+        h->launches += 2;
+    }
     int cur = 0;
     for (int p = 0; p < h->passes; ++p) {
-        SortPass S;
+        SortPass S{};
         S.keys_in = w.keys[cur];
         S.vals_in = w.vals[cur];
         S.keys_out = w.keys[cur ^ 1];
@@ -363,16 +375,26 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
         S.tables = h->d_tables;
         S.n = n;
         S.shift = 8 * p;
-        S.digit_base = w.digit_base + 256 * p;
-        S.base_stride = 256 * h->passes;
-        S.status = w.status + static_cast<size_t>(p) * w.sort_tiles * 256;
-        S.tile_counter = w.tile_counters + p;
-        S.never_set = h->d_never_set;
-        S.force_timeout = (h->flags & CB_DEBUG_FORCE_LOOKBACK_TIMEOUT) && p == 0;
-        S.error = h->d_error;
-        S.timeout_ns = kLookbackTimeoutNs;
-        launch_onesweep(S, w.sp_max_tiles, stream);
-        h->launches += 1;
+        if (lookback) {
+            S.digit_base = w.digit_base + 256 * p;
+            S.base_stride = 256 * h->passes;
+            S.status = w.status + static_cast<size_t>(p) * w.sort_tiles * 256;
+            S.tile_counter = w.tile_counters + p;
+            S.never_set = h->d_never_set;
+            S.force_timeout = (h->flags & CB_DEBUG_FORCE_LOOKBACK_TIMEOUT) && p == 0;
+            S.error = h->d_error;
+            S.timeout_ns = kLookbackTimeoutNs;
+            launch_onesweep(S, w.sp_max_tiles, stream);
+            h->launches += 1;
+        } else {
+            S.table_pos = w.sp_table_pos;
+            S.tile_digits = w.tile_digits;
+            S.seg_sums = w.seg_sums;
+            S.T = h->T;
+            S.segments = w.segments;
+            launch_radix_pass(S, w.sp_max_tiles, stream);
+            h->launches += 4;
+        }
         cur ^= 1;
     }
     record(h, h->ev_bwd[2], stream);

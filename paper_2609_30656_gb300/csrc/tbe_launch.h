@@ -18,10 +18,17 @@ struct SortPass {
     uint32_t* vals_out;
     const struct Chunk* tiles;        // table-aligned tiles of at most 4096 positions
     const int64_t* num_tiles;         // device scalar
-    const int64_t* table_first_tile;  // [T]
+    const int64_t* table_first_tile;  // [T + 1]
     const struct TableDev* tables;
     int64_t n;
     int shift;                   // digit = ((key - row_base_t) >> shift) & 255
+    // reduce-then-scan
+    const int64_t* table_pos;    // [T + 1] first position of each table
+    uint32_t* tile_digits;       // [tiles][256]: digit counts, then first output slots
+    uint32_t* seg_sums;          // [T][segments][256]
+    int T;
+    int segments;                // parts of each table's tiles in the slot scan
+    // single sweep with look-back
     const uint32_t* digit_base;  // [T][stride]: this pass's 256 first output slots per table
     int base_stride;             // passes * 256
     uint32_t* status;            // [tiles * 256], zeroed before the pass
@@ -88,6 +95,10 @@ void launch_sort_hist(const uint32_t* keys, const struct Chunk* tiles, const int
 void launch_sort_bases(const uint32_t* hist, const int64_t* table_pos, int T, int passes,
                        uint32_t* base, cudaStream_t s);
 void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s);
+// Parts per table of the slot scan for a tile bound (about 64 tiles each).
+int radix_segments(int64_t tile_bound, int T);
+// One reduce-then-scan pass: tile counts, segment sums, slots, scatter.
+void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s);
 
 void launch_keygen(const Problem& P, const Plan& Q, const KeyGen& K, bool packed, int64_t chunk_bound,
                    int num_sms, cudaStream_t s);

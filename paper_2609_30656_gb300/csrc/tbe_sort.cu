@@ -3,15 +3,21 @@
 //
 // A table's lookups are contiguous and its row ids are row_base_t + r with
 // r < rows_t, so each table's range is sorted on its own, on the bits of r only
-// (3 passes of 8 bits for tables of up to 16M rows). One streaming kernel counts
-// every pass's digit histogram per table; each pass then reads and writes every
-// pair exactly once ("onesweep"): a block takes the next tile (at most 4096
-// positions of one table) from a counter, ranks its keys by digit (warp match +
-// per-warp counters, stable by position), publishes its per-digit counts, and
-// finds the counts of the table's earlier tiles by a decoupled look-back over
-// their published words. The look-back wait is bounded in time: when it runs
-// out the kernel records CB_ERR_TIMEOUT, publishes anyway so later tiles
-// finish, and writes nothing.
+// (3 passes of 8 bits for tables of up to 16M rows), in tiles of at most 4096
+// positions that never straddle tables. A block ranks its tile's keys by digit
+// (warp match + per-warp counters, stable by position), lays them out by digit
+// in shared memory and writes each digit's run to that digit's slots of the
+// output. The first output slot of each (tile, digit) is found one of two ways:
+//   reduce-then-scan (default): one kernel counts every tile's digits, two
+//     more scan the counts per table (segment sums, then offsets), and the
+//     scatter reads its slots; no block waits on another.
+//   single sweep (CB_SORT_LOOKBACK): one streaming kernel counts every pass's
+//     digit histogram per table; each pass then reads and writes every pair
+//     once, a block publishing its per-digit counts and finding those of the
+//     table's earlier tiles by a decoupled look-back over their published
+//     words. The look-back wait is bounded in time: when it runs out the kernel
+//     records CB_ERR_TIMEOUT, publishes anyway so later tiles finish, and
+//     writes nothing.
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
 
@@ -44,6 +50,90 @@ constexpr int kLookbackWindow = 8;  // predecessor tiles inspected per look-back
 
 __device__ __forceinline__ uint32_t sort_digit(uint32_t key, uint32_t row_base, int shift) {
     return ((key - row_base) >> shift) & (kRadix - 1);
+}
+
+// Stable rank of a tile's keys within each warp; item j of lane l of warp w is
+// tile position w*512 + j*32 + l. The lanes holding one digit in item j find
+// each other (match), their lowest lane adds their number to the warp's
+// counter of that digit and shares the old value. A warp's shared-memory
+// atomics take effect in issue order, so item j's lanes count before item
+// j + 1's, and lanes of one item by lane: the rank follows the position.
+// Positions past the tile count under the extra digit kRadix.
+__device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int tile_count, uint32_t row_base,
+                                          int shift, uint32_t (*sh_warp)[kRadix + 1],
+                                          uint32_t (&rank2)[kSortItems / 2]) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const uint32_t lt_mask = (1u << lane) - 1u;
+#pragma unroll
+    for (int j = 0; j < kSortItems; ++j) {
+        const int local = wid * (32 * kSortItems) + j * 32 + lane;
+        const uint32_t d = local < tile_count ? sort_digit(key[j], row_base, shift) : kRadix;
+        const uint32_t peers = __match_any_sync(kFull, d);
+        const int leader = __ffs(peers) - 1;
+        uint32_t before = 0;
+        if (lane == leader) before = atomicAdd(&sh_warp[wid][d], static_cast<uint32_t>(__popc(peers)));
+        const uint32_t r = __shfl_sync(kFull, before, leader) + __popc(peers & lt_mask);
+        if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;  // two 16-bit ranks per register
+    }
+}
+
+// The tile laid out by digit in shared memory (slot = the digit's tile-local
+// start + the warp's prefix + the rank): every slot first (the counters are
+// read-only here), then the stores.
+__device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], const uint32_t (&val)[kSortItems],
+                                             uint32_t (&rank2)[kSortItems / 2], int tile_count, uint32_t row_base,
+                                             int shift, const uint32_t (*sh_warp)[kRadix + 1],
+                                             const uint32_t* sh_start, uint32_t* sh_keys, uint32_t* sh_vals) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+    for (int j = 0; j < kSortItems; ++j) {
+        const uint32_t dd = sort_digit(key[j], row_base, shift);
+        const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
+        const uint32_t pos = (sh_start[dd] + sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
+        rank2[j >> 1] = (j & 1) ? ((rank2[j >> 1] & 0xffffu) | (pos << 16))
+                                : ((rank2[j >> 1] & 0xffff0000u) | pos);
+    }
+#pragma unroll
+    for (int j = 0; j < kSortItems; ++j) {
+        const int local = wid * (32 * kSortItems) + j * 32 + lane;
+        if (local < tile_count) {
+            const uint32_t pos = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
+            sh_keys[pos] = key[j];
+            sh_vals[pos] = val[j];
+        }
+    }
+}
+
+// Consecutive shared slots of one digit go to consecutive global slots
+// (destination = sh_goff[digit] + slot). Half a tile at a time: its shared
+// reads, its destinations, its stores.
+__device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, uint32_t row_base,
+                                           const int32_t* sh_goff, const uint32_t* sh_keys,
+                                           const uint32_t* sh_vals) {
+    const int tid = threadIdx.x;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        constexpr int kHalf = kSortItems / 2;
+        uint32_t key[kHalf], val[kHalf];
+        int32_t dst[kHalf];
+#pragma unroll
+        for (int j = 0; j < kHalf; ++j) {
+            const int i = tid + (h * kHalf + j) * kSortThreads;
+            key[j] = i < tile_count ? sh_keys[i] : 0u;
+            val[j] = i < tile_count ? sh_vals[i] : 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < kHalf; ++j)
+            dst[j] = sh_goff[sort_digit(key[j], row_base, S.shift)] + tid + (h * kHalf + j) * kSortThreads;
+#pragma unroll
+        for (int j = 0; j < kHalf; ++j) {
+            const int i = tid + (h * kHalf + j) * kSortThreads;
+            if (i < tile_count && dst[j] >= 0 && dst[j] < S.n) {
+                S.keys_out[dst[j]] = key[j];
+                S.vals_out[dst[j]] = val[j];
+            }
+        }
+    }
 }
 
 __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
@@ -84,24 +174,8 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         key[j] = valid ? __ldg(S.keys_in + tile_base + local) : 0u;
         val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
     }
-    // Stable rank within the warp: the lanes holding one digit in item j find
-    // each other (match), their lowest lane adds their number to the warp's
-    // counter of that digit and shares the old value. A warp's shared-memory
-    // atomics take effect in issue order, so item j's lanes count before item
-    // j + 1's, and lanes of one item by lane: the rank follows the position.
-    const uint32_t lt_mask = (1u << lane) - 1u;
-    uint32_t rank2[kSortItems / 2];  // two 16-bit ranks per register
-#pragma unroll
-    for (int j = 0; j < kSortItems; ++j) {
-        const int local = wid * (32 * kSortItems) + j * 32 + lane;
-        const uint32_t d = local < tile_count ? sort_digit(key[j], row_base, S.shift) : kRadix;
-        const uint32_t peers = __match_any_sync(kFull, d);
-        const int leader = __ffs(peers) - 1;
-        uint32_t before = 0;
-        if (lane == leader) before = atomicAdd(&sh_warp[wid][d], static_cast<uint32_t>(__popc(peers)));
-        const uint32_t r = __shfl_sync(kFull, before, leader) + __popc(peers & lt_mask);
-        if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;
-    }
+    uint32_t rank2[kSortItems / 2];
+    rank_tile(key, tile_count, row_base, S.shift, sh_warp, rank2);
     __syncthreads();
 
     // Thread d: per-warp exclusive prefix and the tile's count of digit d.
@@ -176,52 +250,157 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         static_cast<int64_t>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) + excl - start);
     __syncthreads();
 
-    // Scatter into shared memory in tile-sorted order: every slot first (the
-    // counters are read-only here), then the stores.
+    scatter_tile(key, val, rank2, tile_count, row_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
+    __syncthreads();
+    if (sh_abort) return;
+    write_tile(S, tile_count, row_base, sh_goff, sh_keys, sh_vals);
+}
+
+// ---------------------------------------------------------------- reduce-then-scan
+
+// (a) Digit counts of every tile of this pass: 16 keys per thread, shared
+// counters (their order does not matter here).
+__global__ void __launch_bounds__(kSortThreads) radix_count_kernel(const SortPass S) {
+    __shared__ uint32_t sh[kRadix];
+    const int64_t tile = blockIdx.x;
+    if (tile >= *S.num_tiles) return;  // the grid is an upper bound on the tiles
+    const int tid = threadIdx.x;
+    sh[tid] = 0;
+    const Chunk tc = S.tiles[tile];
+    const int count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tc.k0));
+    const uint32_t rb = static_cast<uint32_t>(S.tables[tc.table].row_base);
+    uint32_t k[kSortItems];
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
-        const uint32_t dd = sort_digit(key[j], row_base, S.shift);
-        const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
-        const uint32_t pos = (sh_start[dd] + sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
-        rank2[j >> 1] = (j & 1) ? ((rank2[j >> 1] & 0xffffu) | (pos << 16))
-                                : ((rank2[j >> 1] & 0xffff0000u) | pos);
+        const int i = tid + j * kSortThreads;
+        k[j] = i < count ? __ldg(S.keys_in + tc.k0 + i) : 0u;
     }
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < kSortItems; ++j)
+        if (tid + j * kSortThreads < count) atomicAdd(&sh[sort_digit(k[j], rb, S.shift)], 1u);
+    __syncthreads();
+    S.tile_digits[tile * kRadix + tid] = sh[tid];
+}
+
+// Table t's tiles [f, e) cut into S.segments equal parts; part s is [a, b).
+__device__ __forceinline__ void segment_range(const SortPass& S, int t, int s, int64_t* a, int64_t* b) {
+    const int64_t f = S.table_first_tile[t], e = S.table_first_tile[t + 1];
+    const int64_t per = (e - f + S.segments - 1) / S.segments;
+    *a = min64(f + s * per, e);
+    *b = min64(*a + per, e);
+}
+
+// (b) Per (table, segment) block, thread d: the segment's count of digit d.
+__global__ void __launch_bounds__(kRadix) radix_segsum_kernel(const SortPass S) {
+    const int t = blockIdx.x / S.segments, sg = blockIdx.x % S.segments, d = threadIdx.x;
+    int64_t a, b;
+    segment_range(S, t, sg, &a, &b);
+    const uint32_t* c = S.tile_digits + d;
+    uint32_t sum = 0;
+    int64_t k = a;
+    for (; k + 8 <= b; k += 8) {
+        uint32_t v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = c[(k + u) * kRadix];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) sum += v[u];
+    }
+    for (; k < b; ++k) sum += c[k * kRadix];
+    S.seg_sums[(static_cast<int64_t>(t) * S.segments + sg) * kRadix + d] = sum;
+}
+
+// (c) Per (table, segment) block, thread d: the first output slot of digit d in
+// each of the segment's tiles, replacing its count. The slots of digit d in
+// table t start at the table's first position plus the table's counts of the
+// smaller digits; within the digit, tiles (and segments) keep their order.
+__global__ void __launch_bounds__(kRadix) radix_offsets_kernel(const SortPass S) {
+    __shared__ int64_t sh_scan[33];
+    const int t = blockIdx.x / S.segments, sg = blockIdx.x % S.segments, d = threadIdx.x;
+    const uint32_t* ss = S.seg_sums + static_cast<int64_t>(t) * S.segments * kRadix + d;
+    uint32_t total = 0, before = 0;
+    for (int q = 0; q < S.segments; ++q) {
+        const uint32_t v = ss[q * kRadix];
+        before += q < sg ? v : 0u;
+        total += v;
+    }
+    int64_t all;
+    const int64_t digit_start = block_excl_scan(total, sh_scan, &all);
+    // positions are below 2^30: 32 bits hold every slot
+    uint32_t run = static_cast<uint32_t>(S.table_pos[t] + digit_start) + before;
+    int64_t a, b;
+    segment_range(S, t, sg, &a, &b);
+    uint32_t* c = S.tile_digits + d;
+    int64_t k = a;
+    for (; k + 8 <= b; k += 8) {
+        uint32_t v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = c[(k + u) * kRadix];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            c[(k + u) * kRadix] = run;
+            run += v[u];
+        }
+    }
+    for (; k < b; ++k) {
+        const uint32_t v = c[k * kRadix];
+        c[k * kRadix] = run;
+        run += v;
+    }
+}
+
+// (d) The scatter of tile blockIdx.x: the ranking of the single-sweep kernel,
+// with the first output slot of every digit read from (c).
+__global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const SortPass S) {
+    extern __shared__ __align__(16) uint32_t sh_dyn[];
+    uint32_t* sh_keys = sh_dyn;                            // tile-sorted keys
+    uint32_t* sh_vals = sh_dyn + kSortTile;                // tile-sorted payloads
+    __shared__ uint32_t sh_warp[kSortWarps][kRadix + 1];   // per-warp counts, then prefixes
+                                                           // (slot kRadix: positions past the tile)
+    __shared__ uint32_t sh_start[kRadix];                  // tile-local start of each digit
+    __shared__ int32_t sh_goff[kRadix];                    // global destination - local index
+    __shared__ int64_t sh_scan[33];
+
+    const int64_t tile = blockIdx.x;
+    if (tile >= *S.num_tiles) return;  // the grid is an upper bound on the tiles
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    for (int i = tid; i < kSortWarps * (kRadix + 1); i += kSortThreads) (&sh_warp[0][0])[i] = 0;
+    const uint32_t slot = S.tile_digits[tile * kRadix + tid];  // digit tid's first output slot
+    const Chunk tc = S.tiles[tile];
+    const int64_t tile_base = tc.k0;
+    const int tile_count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tile_base));
+    const uint32_t row_base = static_cast<uint32_t>(S.tables[tc.table].row_base);
+    uint32_t key[kSortItems], val[kSortItems];
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
-        if (local < tile_count) {
-            const uint32_t pos = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
-            sh_keys[pos] = key[j];
-            sh_vals[pos] = val[j];
-        }
+        const bool valid = local < tile_count;
+        key[j] = valid ? __ldg(S.keys_in + tile_base + local) : 0u;
+        val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
     }
     __syncthreads();
-    if (sh_abort) return;
-    // Consecutive shared slots of one digit go to consecutive global slots.
-    // Half a tile at a time: its shared reads, its destinations, its stores.
+    uint32_t rank2[kSortItems / 2];
+    rank_tile(key, tile_count, row_base, S.shift, sh_warp, rank2);
+    __syncthreads();
+    const int d = tid;
+    uint32_t count = 0;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        constexpr int kHalf = kSortItems / 2;
-        int32_t dst[kHalf];
-#pragma unroll
-        for (int j = 0; j < kHalf; ++j) {
-            const int i = tid + (h * kHalf + j) * kSortThreads;
-            key[j] = i < tile_count ? sh_keys[i] : 0u;
-            val[j] = i < tile_count ? sh_vals[i] : 0u;
-        }
-#pragma unroll
-        for (int j = 0; j < kHalf; ++j)
-            dst[j] = sh_goff[sort_digit(key[j], row_base, S.shift)] + tid + (h * kHalf + j) * kSortThreads;
-#pragma unroll
-        for (int j = 0; j < kHalf; ++j) {
-            const int i = tid + (h * kHalf + j) * kSortThreads;
-            if (i < tile_count && dst[j] >= 0 && dst[j] < S.n) {
-                S.keys_out[dst[j]] = key[j];
-                S.vals_out[dst[j]] = val[j];
-            }
-        }
+    for (int w = 0; w < kSortWarps; ++w) {
+        const uint32_t c = sh_warp[w][d];
+        sh_warp[w][d] = count;
+        count += c;
     }
+    int64_t total;
+    const int64_t start = block_excl_scan(count, sh_scan, &total);
+    sh_start[d] = static_cast<uint32_t>(start);
+    sh_goff[d] = static_cast<int32_t>(static_cast<int64_t>(slot) - start);
+    __syncthreads();
+    scatter_tile(key, val, rank2, tile_count, row_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
+    __syncthreads();
+    write_tile(S, tile_count, row_base, sh_goff, sh_keys, sh_vals);
 }
+
+// ---------------------------------------------------------------- single sweep
 
 // Digit histograms of every pass, per table. Each block streams a contiguous
 // range of tiles, so its shared histogram changes table only a few times.
@@ -298,6 +477,20 @@ void launch_sort_bases(const uint32_t* hist, const int64_t* table_pos, int T, in
 }
 
 constexpr int kSortDynSmem = 2 * kSortTile * sizeof(uint32_t);  // 32 KB
+
+int radix_segments(int64_t tile_bound, int T) {
+    const int64_t per_table = tile_bound / max64(T, 1) + 1;
+    return static_cast<int>(min64(max64((per_table + 63) / 64, 1), 1024));
+}
+
+void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
+    const unsigned grid = static_cast<unsigned>(max64(tile_bound, 1));
+    const unsigned parts = static_cast<unsigned>(S.T) * static_cast<unsigned>(S.segments);
+    radix_count_kernel<<<grid, kSortThreads, 0, s>>>(S);
+    radix_segsum_kernel<<<parts, kRadix, 0, s>>>(S);
+    radix_offsets_kernel<<<parts, kRadix, 0, s>>>(S);
+    radix_scatter_kernel<<<grid, kSortThreads, kSortDynSmem, s>>>(S);
+}
 
 void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     static bool configured = false;

@@ -20,7 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libcb_tbe.so")
 
 CB_OK, CB_ERR_INVALID_ARG, CB_ERR_INDEX_OOB, CB_ERR_BAD_OFFSETS = 0, 1, 2, 3
 CB_ERR_CAPACITY, CB_ERR_OOM, CB_ERR_CUDA, CB_ERR_TIMEOUT = 4, 5, 6, 7
-CB_VALIDATE, CB_TIMING, CB_DEBUG_FORCE_LOOKBACK_TIMEOUT = 0x1, 0x2, 0x100
+CB_VALIDATE, CB_TIMING, CB_DEBUG_FORCE_LOOKBACK_TIMEOUT, CB_SORT_LOOKBACK = 0x1, 0x2, 0x100, 0x200
 CB_OUT_F16, CB_OUT_BF16 = 0x4, 0x8
 _OUT_FLAGS = {torch.float32: 0, torch.float16: CB_OUT_F16, torch.bfloat16: CB_OUT_BF16}
 _DTYPES = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2}

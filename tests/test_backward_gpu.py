@@ -114,6 +114,28 @@ def test_bitwise_deterministic():
     assert torch.equal(a.unique_ids[:a.num_unique], b.unique_ids[:b.num_unique])
 
 
+@pytest.mark.parametrize("weighted,mean", [(False, False), (True, True)])
+def test_both_radix_pass_forms_give_the_same_bits(weighted, mean):
+    # Reduce-then-scan and single-sweep passes are both stable sorts of the
+    # same pairs: the sorted order, and so every gradient bit, must agree.
+    # Rows > 2^16 (three passes), hot rows (Zipf) and tables of 1-2 tiles.
+    from paper_2609_30656_gb300.tbe import CB_SORT_LOOKBACK
+    tables, ind, off, w = random_problem(37, dims=(16, 64, 128), rows=(3, 70000, 300000), batch=700,
+                                         max_len=120, weighted=weighted, empty_frac=0.1)
+    rows, dims = table_meta(tables)
+    go = torch.randn(700, int(dims.sum()), generator=torch.Generator().manual_seed(38))
+    args = (ind.to(DEV), off.to(DEV), go.to(DEV), None if w is None else w.to(DEV))
+    pooling = "mean" if mean else "sum"
+    a = _tbe(tables, pooling).backward(*args)
+    b = _tbe(tables, pooling, extra_flags=CB_SORT_LOOKBACK).backward(*args)
+    torch.cuda.synchronize()
+    assert a.num_unique == b.num_unique and a.num_floats == b.num_floats
+    assert torch.equal(a.unique_ids[:a.num_unique], b.unique_ids[:b.num_unique])
+    assert torch.equal(a.grads[:a.num_floats], b.grads[:b.num_floats])
+    res, scale = backward_reference(rows, dims, 700, ind, off, go, w, mean)
+    assert_backward_matches(a, res, scale)
+
+
 def test_forced_lookback_timeout_returns_an_error_and_the_context_survives():
     from paper_2609_30656_gb300.tbe import CB_DEBUG_FORCE_LOOKBACK_TIMEOUT, CB_ERR_TIMEOUT
     # Enough lookups for several radix tiles; tile 1 waits on a word nothing writes.
