@@ -24,6 +24,11 @@ constexpr int kRleTile = kRleThreads * kRleItems;
 
 // ---------------------------------------------------------------- (1) keys
 
+// A warp walks one chunk kKeygenSteps x 32 lookups at a time: the indices (and
+// weights) of all the steps are loaded first, so that many loads are in flight
+// per warp, then each step finds its lanes' bags and writes.
+constexpr int kKeygenSteps = 8;
+
 template <bool PACKED>
 __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q, KeyGen K) {
     const int lane = threadIdx.x & 31;
@@ -32,28 +37,39 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];
+        const int64_t rows = td.rows, row_base = td.row_base;
         const int64_t k0 = ch.k0, k1 = ch.k0 + (ch.len & 0x7fffffffu);
         const int64_t bag_lo = static_cast<int64_t>(t) * P.B, bag_hi = bag_lo + P.B;
         BagWindow W = bag_window(P, ch.first, bag_hi, lane);
-        for (int64_t base = k0; base < k1; base += 32) {
-            const int64_t q = base + lane;
-            const bool valid = q < k1;
-            int64_t my_bag, my_s, my_e;
-            find_bag(P, W, q, valid, lane, my_bag, my_s, my_e);
-            if (valid) {
+        for (int64_t base = k0; base < k1; base += 32 * kKeygenSteps) {
+            int64_t idx[kKeygenSteps];
+            float wt[kKeygenSteps];
+#pragma unroll
+            for (int u = 0; u < kKeygenSteps; ++u) {
+                const int64_t q = base + 32 * u + lane;
+                idx[u] = q < k1 ? load_index(P.indices, q, P.is32) : 0;
+                wt[u] = PACKED && P.weights && q < k1 ? __ldg(P.weights + q) : 1.f;
+            }
+#pragma unroll
+            for (int u = 0; u < kKeygenSteps; ++u) {
+                const int64_t q = base + 32 * u + lane;
+                if (base + 32 * u >= k1) break;  // warp-uniform
+                const bool valid = q < k1;
+                int64_t my_bag, my_s, my_e;
+                find_bag(P, W, q, valid, lane, my_bag, my_s, my_e);
+                if (!valid) continue;
                 if (my_bag >= bag_hi) {  // only reachable with malformed offsets
                     set_error(P.error, CB_ERR_BAD_OFFSETS);
                     my_bag = bag_hi - 1;
                 }
-                int64_t r = load_index(P.indices, q, P.is32);
-                if (r < 0 || r >= td.rows) {
+                int64_t r = idx[u];
+                if (r < 0 || r >= rows) {
                     set_error(P.error, CB_ERR_INDEX_OOB);
-                    r = r < 0 ? 0 : td.rows - 1;
+                    r = r < 0 ? 0 : rows - 1;
                 }
-                const uint32_t key = static_cast<uint32_t>(td.row_base + r);
-                K.keys[q] = key;
+                K.keys[q] = static_cast<uint32_t>(row_base + r);
                 if (PACKED) {
-                    float c = P.weights ? __ldg(P.weights + q) : 1.f;
+                    float c = wt[u];
                     if (P.mean && my_e > my_s) c = c / static_cast<float>(my_e - my_s);
                     K.vals[q] = static_cast<uint32_t>(q);
                     K.packed[q] = make_uint2(static_cast<uint32_t>(my_bag), __float_as_uint(c));
