@@ -95,7 +95,7 @@ void launch_sort_hist(const uint32_t* keys, const struct Chunk* tiles, const int
 void launch_sort_bases(const uint32_t* hist, const int64_t* table_pos, int T, int passes,
                        uint32_t* base, cudaStream_t s);
 void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s);
-// Parts per table of the slot scan for a tile bound (about 64 tiles each).
+// Parts per table of the slot scan for a tile bound (about 16 tiles each).
 int radix_segments(int64_t tile_bound, int T);
 // One reduce-then-scan pass: tile counts, segment sums, slots, scatter.
 void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s);

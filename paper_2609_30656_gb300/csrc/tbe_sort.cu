@@ -480,7 +480,7 @@ constexpr int kSortDynSmem = 2 * kSortTile * sizeof(uint32_t);  // 32 KB
 
 int radix_segments(int64_t tile_bound, int T) {
     const int64_t per_table = tile_bound / max64(T, 1) + 1;
-    return static_cast<int>(min64(max64((per_table + 63) / 64, 1), 1024));
+    return static_cast<int>(min64(max64((per_table + 15) / 16, 1), 1024));
 }
 
 void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
