@@ -370,7 +370,7 @@ void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const v
     } else if (apply) {
         launch_bwd_reduce_f32_apply(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
     } else {
-        launch_bwd_reduce_t<CB_F32, false>(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
+        launch_bwd_reduce_f32(P, Q, O, grad_out, cls, vpl, gc, packed, chunk_bound, num_sms, s);
     }
 }
 

@@ -111,6 +111,8 @@ void launch_bwd_finalize(const Problem& P, const BwdOut& O, cudaStream_t s);
 void launch_bwd_reduce(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out, int cls,
                        int vpl, int gc, bool packed, bool apply, int64_t chunk_bound, int num_sms,
                        cudaStream_t s);
+void launch_bwd_reduce_f32(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out, int cls,
+                           int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms, cudaStream_t s);
 void launch_bwd_reduce_f32_apply(const Problem& P, const Plan& Q, const BwdOut& O, const void* grad_out,
                                  int cls, int vpl, int gc, bool packed, int64_t chunk_bound, int num_sms,
                                  cudaStream_t s);

@@ -93,6 +93,8 @@ def test_clock_summary_parsing():
 def test_traffic_is_null_unless_recorded_for_this_source(tmp_path, monkeypatch):
     assert bench.recorded_traffic("fwd.gather", "no-such-workload") is None
     assert len(bench.kernel_source_hash()) == 16
+    for k in bench.KERNEL_SOURCES:  # every listed source exists
+        assert len(bench.kernel_source_hash(k)) == 16
 
 
 def _free_port():
