@@ -8,7 +8,7 @@ leaves (Sec. IV.A.2 on inter_arch.deep_fm.dense_module), and a parent that could
 not be profiled is estimated from its children (Sec. III, recursive profiling).
 
 Here the components are the library's kernels grouped by direction
-(``step / forward / fwd.gather`` ...). A leaf carries a measured latency and its
+(``run / step / forward / fwd.gather`` ...). A leaf carries a measured latency and its
 algorithmic bytes and FLOPs; a parent without a latency of its own gets the sum
 of its children's (the kernels run one after another on one stream). Rates of a
 parent are latency-weighted means of its leaves' rates, which equal its total
@@ -116,11 +116,13 @@ def to_markdown(root: Component, peak_gbs: float, peak_tflops: float, title: str
 def step_tree(comp_ms: dict[str, float], comp_bytes: dict[str, float], comp_flops: dict[str, float],
               table_mb: float, workspace_mb: float, extra: dict[str, tuple[float, float, float]] | None = None
               ) -> Component:
-    """The step's tree from per-component latency, bytes and FLOPs. `extra` maps further
-    leaves under ``next`` (name -> (ms, bytes, flops))."""
-    root = Component("step", size_mb=table_mb + workspace_mb)
+    """The run's tree from per-component latency, bytes and FLOPs: ``run / step /
+    {forward, backward} / <kernels>``, and beside the step ``run / next / <extra>``
+    for the further rows timed on their own (name -> (ms, bytes, flops))."""
+    root = Component("run")
+    step = root.add(Component("step", size_mb=table_mb + workspace_mb))
     for direction, prefix in (("forward", "fwd."), ("backward", "bwd.")):
-        node = root.add(Component(direction, size_mb=table_mb))
+        node = step.add(Component(direction, size_mb=table_mb))
         for name in comp_ms:
             if name.startswith(prefix):
                 node.add(Component(name, comp_ms[name], comp_bytes.get(name, 0.0),

@@ -147,11 +147,14 @@ def test_report_written_from_measured_components(tmp_path):
     bench.write_report(str(tmp_path / "r"), w, line, comp_ms, comp_bytes, [c], [[3, 1]], 1000.0)
     doc = json.loads((tmp_path / "r.json").read_text())
     names = [r["component"] for r in doc["components"]]
-    assert names[:3] == ["step", "step/forward", "step/forward/fwd.prep"]
-    assert "step/next/fm.forward" in names and "step/next/backward_apply.sgd" in names
-    gather = doc["components"][names.index("step/forward/fwd.gather")]
+    assert names[:4] == ["run", "run/step", "run/step/forward", "run/step/forward/fwd.prep"]
+    assert "run/next/fm.forward" in names and "run/next/backward_apply.sgd" in names
+    gather = doc["components"][names.index("run/step/forward/fwd.gather")]
     assert gather["est_avg_bw_gbs"] == pytest.approx(6000.0)  # 6 GB in 1 ms
-    bwd = doc["components"][names.index("step/backward")]
+    bwd = doc["components"][names.index("run/step/backward")]
     assert bwd["latency_ms"] == pytest.approx(2.8) and bwd["est_avg_bw_gbs"] == pytest.approx(8e9 / 2.8e-3 / 1e9, abs=0.1)
-    assert doc["components"][0]["latency_ms"] == 4.0
+    step = doc["components"][names.index("run/step")]
+    assert step["latency_ms"] == 4.0 and step["measured"]
+    # the step's rate covers its own kernels: (6 + 8) GB over their 3.82 ms
+    assert step["est_avg_bw_gbs"] == pytest.approx(14e9 / 3.82e-3 / 1e9, abs=0.1)
     assert "| fwd.gather |" in (tmp_path / "r.md").read_text().replace("&nbsp;", "")

@@ -54,10 +54,14 @@ def test_step_tree_from_component_timings():
           "bwd.sort": 4.0, "bwd.rle": 0.4, "bwd.reduce": 8.0}
     t = report.step_tree(ms, {"fwd.gather": 6e9}, {}, table_mb=100.0, workspace_mb=10.0,
                          extra={"fm.forward": (0.5, 3e9, 1e9)})
-    assert [c.name for c in t.children] == ["forward", "backward", "next"]
-    assert [c.name for c in t.children[0].children] == ["fwd.prep", "fwd.gather", "fwd.fixup"]
-    assert report.latency(t.children[1]) == pytest.approx(13.4)
-    assert t.size_mb == 110.0
+    assert [c.name for c in t.children] == ["step", "next"]
+    step = t.children[0]
+    assert [c.name for c in step.children] == ["forward", "backward"]
+    assert [c.name for c in step.children[0].children] == ["fwd.prep", "fwd.gather", "fwd.fixup"]
+    assert report.latency(step.children[1]) == pytest.approx(13.4)
+    assert step.size_mb == 110.0
+    # the step's rates come from its own kernels only, not from the rows beside it
+    assert report.bandwidth_gbs(step) == pytest.approx(6e9 / (sum(ms.values()) * 1e-3) / 1e9)
 
 
 def test_component_flops_by_hand():
