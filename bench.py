@@ -703,7 +703,7 @@ def run_e2e(args, m, w, batches, grads_out, g, out, dev, world):
     h_w = None if b.weights is None else b.weights.cpu().pin_memory()
     h_go = go.cpu().pin_memory()
     h_res = torch.empty(2 + w.num_tables + 1, dtype=torch.int64).pin_memory()
-    steps = max(2, min(args.steps, args.e2e_steps))
+    steps = max(2, args.steps if args.e2e_steps is None else min(args.steps, args.e2e_steps))
     bytes_in = (h_ind.numel() * 8 + h_off.numel() * 8 + (0 if h_w is None else h_w.numel() * 4)
                 + h_go.numel() * 4)
     bytes_out = h_res.numel() * 8
@@ -864,7 +864,8 @@ def main(argv=None):
     ap.add_argument("--rows", type=int, default=None,
                     help="cap every table's rows (a smaller case for profiling; same lengths and batch)")
     ap.add_argument("--rotate", type=int, default=4)
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=None,
+                    help="steps of the end-to-end timing (default: --steps)")
     ap.add_argument("--cpu-tables", type=int, default=32)
     ap.add_argument("--ref-tables", type=int, default=2)
     ap.add_argument("--ref-budget-s", type=float, default=150.0)
