@@ -24,6 +24,60 @@ constexpr int kRleTile = kRleThreads * kRleItems;
 
 // ---------------------------------------------------------------- (1) keys
 
+// The bag of each lookup, from a window of 32 bag ends held one per lane, in
+// positions relative to the chunk start: every position is below 2^30, so these
+// are exact in 32 bits (saturated, for malformed offsets, well inside the
+// sentinel kPastTable that marks ends past the table's last bag).
+constexpr int32_t kPastTable = INT32_MAX;
+
+__device__ __forceinline__ int32_t rel32(int64_t x, int64_t k0) {
+    const int64_t r = x - k0;
+    return static_cast<int32_t>(r < -(int64_t(1) << 30) ? -(int64_t(1) << 30)
+                                                        : (r > (int64_t(1) << 30) ? (int64_t(1) << 30) : r));
+}
+
+struct BagWindow32 {
+    int64_t win;        // first bag of the window
+    int32_t win_start;  // start of bag win
+    int32_t my_end;     // end of bag win + lane
+};
+
+__device__ __forceinline__ BagWindow32 bag_window32(const Problem& P, int64_t first, int64_t bag_hi,
+                                                    int64_t k0, int lane) {
+    BagWindow32 W;
+    W.win = first;
+    W.win_start = first < bag_hi ? rel32(load_index(P.offsets, first, P.is32), k0) : kPastTable;
+    W.my_end = first + lane < bag_hi ? rel32(load_index(P.offsets, first + lane + 1, P.is32), k0) : kPastTable;
+    return W;
+}
+
+// Every lane calls this with its relative position q; the window moves forward
+// 32 bags at a time until every valid lane has its bag (bag = -1 otherwise).
+__device__ __forceinline__ void find_bag32(const Problem& P, BagWindow32& W, int64_t bag_hi, int64_t k0,
+                                           int32_t q, bool valid, int lane, int64_t& bag, int32_t& s,
+                                           int32_t& e) {
+    bag = -1;
+    s = e = 0;
+    while (true) {
+        int cnt = 0;  // ends at or before q in the window
+#pragma unroll
+        for (int b = 16; b >= 1; b >>= 1)
+            if (__shfl_sync(kFull, W.my_end, cnt + b - 1) <= q) cnt += b;
+        if (__shfl_sync(kFull, W.my_end, 31) <= q) cnt = 32;
+        const int32_t e_sel = __shfl_sync(kFull, W.my_end, cnt < 32 ? cnt : 31);
+        const int32_t s_sel = __shfl_sync(kFull, W.my_end, cnt > 0 ? cnt - 1 : 0);
+        if (valid && bag < 0 && cnt < 32) {
+            bag = W.win + cnt;
+            e = e_sel;
+            s = cnt > 0 ? s_sel : W.win_start;
+        }
+        if (!__any_sync(kFull, valid && bag < 0)) break;
+        W.win_start = __shfl_sync(kFull, W.my_end, 31);
+        W.win += 32;
+        W.my_end = W.win + lane < bag_hi ? rel32(load_index(P.offsets, W.win + lane + 1, P.is32), k0) : kPastTable;
+    }
+}
+
 // A warp walks one chunk kKeygenSteps x 32 lookups at a time: the indices (and
 // weights) of all the steps are loaded first, so that many loads are in flight
 // per warp, then each step finds its lanes' bags and writes.
@@ -38,25 +92,29 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
         const int t = ch.table;
         const TableDev& td = P.tables[t];
         const int64_t rows = td.rows, row_base = td.row_base;
-        const int64_t k0 = ch.k0, k1 = ch.k0 + (ch.len & 0x7fffffffu);
+        const int64_t k0 = ch.k0;
+        const int32_t len = static_cast<int32_t>(ch.len & 0x7fffffffu);
         const int64_t bag_lo = static_cast<int64_t>(t) * P.B, bag_hi = bag_lo + P.B;
-        BagWindow W = bag_window(P, ch.first, bag_hi, lane);
-        for (int64_t base = k0; base < k1; base += 32 * kKeygenSteps) {
+        uint32_t* keys = K.keys + k0;
+        uint32_t* vals = K.vals + k0;
+        BagWindow32 W = bag_window32(P, ch.first, bag_hi, k0, lane);
+        for (int32_t base = 0; base < len; base += 32 * kKeygenSteps) {
             int64_t idx[kKeygenSteps];
             float wt[kKeygenSteps];
 #pragma unroll
             for (int u = 0; u < kKeygenSteps; ++u) {
-                const int64_t q = base + 32 * u + lane;
-                idx[u] = q < k1 ? load_index(P.indices, q, P.is32) : 0;
-                wt[u] = PACKED && P.weights && q < k1 ? __ldg(P.weights + q) : 1.f;
+                const int32_t q = base + 32 * u + lane;
+                idx[u] = q < len ? load_index(P.indices, k0 + q, P.is32) : 0;
+                wt[u] = PACKED && P.weights && q < len ? __ldg(P.weights + k0 + q) : 1.f;
             }
 #pragma unroll
             for (int u = 0; u < kKeygenSteps; ++u) {
-                const int64_t q = base + 32 * u + lane;
-                if (base + 32 * u >= k1) break;  // warp-uniform
-                const bool valid = q < k1;
-                int64_t my_bag, my_s, my_e;
-                find_bag(P, W, q, valid, lane, my_bag, my_s, my_e);
+                const int32_t q = base + 32 * u + lane;
+                if (base + 32 * u >= len) break;  // warp-uniform
+                const bool valid = q < len;
+                int64_t my_bag;
+                int32_t my_s, my_e;
+                find_bag32(P, W, bag_hi, k0, q, valid, lane, my_bag, my_s, my_e);
                 if (!valid) continue;
                 if (my_bag >= bag_hi) {  // only reachable with malformed offsets
                     set_error(P.error, CB_ERR_BAD_OFFSETS);
@@ -67,14 +125,14 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
                     set_error(P.error, CB_ERR_INDEX_OOB);
                     r = r < 0 ? 0 : rows - 1;
                 }
-                K.keys[q] = static_cast<uint32_t>(row_base + r);
+                keys[q] = static_cast<uint32_t>(row_base + r);
                 if (PACKED) {
                     float c = wt[u];
                     if (P.mean && my_e > my_s) c = c / static_cast<float>(my_e - my_s);
-                    K.vals[q] = static_cast<uint32_t>(q);
-                    K.packed[q] = make_uint2(static_cast<uint32_t>(my_bag), __float_as_uint(c));
+                    vals[q] = static_cast<uint32_t>(k0 + q);
+                    K.packed[k0 + q] = make_uint2(static_cast<uint32_t>(my_bag), __float_as_uint(c));
                 } else {
-                    K.vals[q] = static_cast<uint32_t>(my_bag);
+                    vals[q] = static_cast<uint32_t>(my_bag);
                 }
             }
         }
