@@ -183,23 +183,23 @@ __global__ void __launch_bounds__(kRleThreads) rle_count_kernel(const uint32_t* 
     if (threadIdx.x == 0) tile_heads[blockIdx.x] = total;
 }
 
+// One block: thread i sums a contiguous range of the tile counts, one block
+// scan, then the thread writes its range's exclusive prefixes.
 __global__ void __launch_bounds__(1024) rle_scan_kernel(const int64_t* tile_heads, int64_t tiles,
                                                         int64_t* tile_base, int64_t* num_unique) {
     __shared__ int64_t sh[33];
-    __shared__ int64_t running;
-    if (threadIdx.x == 0) running = 0;
-    __syncthreads();
-    for (int64_t i0 = 0; i0 < tiles; i0 += blockDim.x) {
-        const int64_t i = i0 + threadIdx.x;
-        const int64_t c = i < tiles ? tile_heads[i] : 0;
-        int64_t total;
-        const int64_t ex = block_excl_scan(c, sh, &total);
-        if (i < tiles) tile_base[i] = running + ex;
-        __syncthreads();
-        if (threadIdx.x == 0) running += total;
-        __syncthreads();
+    const int64_t per = (tiles + blockDim.x - 1) / blockDim.x;
+    const int64_t lo = min64(static_cast<int64_t>(threadIdx.x) * per, tiles), hi = min64(lo + per, tiles);
+    int64_t sum = 0;
+    for (int64_t i = lo; i < hi; ++i) sum += tile_heads[i];
+    int64_t total;
+    int64_t run = block_excl_scan(sum, sh, &total);
+    for (int64_t i = lo; i < hi; ++i) {
+        const int64_t c = tile_heads[i];
+        tile_base[i] = run;
+        run += c;
     }
-    if (threadIdx.x == 0) *num_unique = running;
+    if (threadIdx.x == 0) *num_unique = total;
 }
 
 __global__ void __launch_bounds__(kRleThreads) rle_write_kernel(const uint32_t* keys, int64_t n,
@@ -314,9 +314,10 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_fixup_kernel(const __grid_co
     }
 }
 
-// One heavy run per block: warp w adds pieces w, w + 8, ... (lanes own columns),
-// then the warps' partial sums meet in shared memory in warp order, after the
-// tail piece. The order is fixed, so the result is deterministic.
+// One heavy run per block: warp w adds pieces w, w + 8, ... (lanes own columns;
+// fp32 groups folded into fp64), then the warps' partial sums meet in shared
+// memory in warp order, after the tail piece. The order is fixed, so the result
+// is deterministic.
 __global__ void __launch_bounds__(kWarpThreads) bwd_heavy_kernel(const __grid_constant__ Problem P,
                                                                  const __grid_constant__ Plan Q,
                                                                  const __grid_constant__ BwdOut O) {
@@ -333,14 +334,7 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_heavy_kernel(const __grid_co
         const float* head = Q.carry_head + (j + 1) * P.dmax;
         for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {
             double acc[4] = {0.0, 0.0, 0.0, 0.0};
-#pragma unroll 8
-            for (int64_t i = w; i < m; i += kWarps) {
-                const float4 v = *reinterpret_cast<const float4*>(head + i * P.dmax + x0);
-                acc[0] += v.x;
-                acc[1] += v.y;
-                acc[2] += v.z;
-                acc[3] += v.w;
-            }
+            add_pieces(head, w, kWarps, m, P.dmax, x0, acc);
             for (int x = 0; x < 4; ++x) sh[w][x0 + x] = acc[x];
         }
         __syncthreads();

@@ -730,27 +730,57 @@ __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uin
 // A segment that straddles chunks left its tail piece in chunk j and head pieces
 // in the m chunks after it (chunks of a table are contiguous and chunk_len long
 // except the table's last, so m follows from the segment end). The pieces are
-// added in fp64 in a fixed order, so the result is deterministic; `store`
-// receives each group of four columns. Few pieces: lanes own columns and walk
-// the pieces; many pieces (a hot row repeated across hundreds of chunks): lanes
-// own pieces and meet in a butterfly per group of four columns.
+// added in a fixed order, so the result is deterministic; `store` receives each
+// group of four columns in fp64. Up to 32 pieces: lanes own columns and walk the
+// pieces (add_pieces); more pieces (a hot row repeated across hundreds of
+// chunks): lanes own pieces and meet in a butterfly per group of four columns.
+constexpr int kInnerPieces = 16;
+
+// acc (fp64, four columns from x0) += pieces i0, i0 + step, ... below m, each at
+// head + piece * dmax. The pieces are summed in fp32 in groups of kInnerPieces,
+// each group folded into acc: GB300's fp64 adds are scarce (one per piece and
+// column made a heavy-run combine fp64-bound), and an fp32 sum of at most 16
+// pieces rounds within 16u of their absolute sum. Four loads in flight.
+__device__ __forceinline__ void add_pieces(const float* head, int64_t i0, int64_t step, int64_t m, int dmax,
+                                           int x0, double (&acc)[4]) {
+    for (int64_t g = i0; g < m; g += kInnerPieces * step) {
+        const int64_t gend = min64(m, g + kInnerPieces * step);
+        float in[4] = {0.f, 0.f, 0.f, 0.f};
+        int64_t i = g;
+        for (; i + 3 * step < gend; i += 4 * step) {
+            float4 h[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) h[c] = *reinterpret_cast<const float4*>(head + (i + c * step) * dmax + x0);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                in[0] += h[c].x;
+                in[1] += h[c].y;
+                in[2] += h[c].z;
+                in[3] += h[c].w;
+            }
+        }
+        for (; i < gend; i += step) {
+            const float4 h = *reinterpret_cast<const float4*>(head + i * dmax + x0);
+            in[0] += h.x;
+            in[1] += h.y;
+            in[2] += h.z;
+            in[3] += h.w;
+        }
+#pragma unroll
+        for (int x = 0; x < 4; ++x) acc[x] += in[x];
+    }
+}
+
 template <class Store>
 __device__ __forceinline__ void combine_pieces(const Plan& Q, int64_t j, int64_t m, int dim,
                                                int dmax, int lane, Store store) {
     const float* tail = Q.carry_tail + j * dmax;
     const float* head = Q.carry_head + (j + 1) * dmax;
-    if (m <= 16) {
+    if (m <= 32) {
         for (int x0 = lane * 4; x0 < dim; x0 += 128) {
             const float4 a = *reinterpret_cast<const float4*>(tail + x0);
             double acc[4] = {a.x, a.y, a.z, a.w};
-#pragma unroll 4
-            for (int64_t i = 0; i < m; ++i) {
-                const float4 h = *reinterpret_cast<const float4*>(head + i * dmax + x0);
-                acc[0] += h.x;
-                acc[1] += h.y;
-                acc[2] += h.z;
-                acc[3] += h.w;
-            }
+            add_pieces(head, 0, 1, m, dmax, x0, acc);
             store(x0, acc);
         }
         return;
