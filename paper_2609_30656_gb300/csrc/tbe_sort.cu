@@ -52,6 +52,18 @@ __device__ __forceinline__ uint32_t sort_digit(uint32_t key, uint32_t row_base, 
     return ((key - row_base) >> shift) & (kRadix - 1);
 }
 
+// *p += v in the lanes where `on`, returning the old value there (0 elsewhere):
+// one predicated shared-memory atomic, with no branch around it.
+__device__ __forceinline__ uint32_t shared_add_if(uint32_t* p, uint32_t v, bool on) {
+    uint32_t old = 0;
+    asm volatile(
+        "{\n\t.reg .pred q;\n\tsetp.ne.u32 q, %1, 0;\n\t@q atom.shared.add.u32 %0, [%2], %3;\n\t}"
+        : "+r"(old)
+        : "r"(static_cast<uint32_t>(on)), "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))), "r"(v)
+        : "memory");
+    return old;
+}
+
 // Stable rank of a tile's keys within each warp; item j of lane l of warp w is
 // tile position w*512 + j*32 + l. The lanes holding one digit in item j find
 // each other (match), their lowest lane adds their number to the warp's
@@ -70,8 +82,8 @@ __device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int
         const uint32_t d = local < tile_count ? sort_digit(key[j], row_base, shift) : kRadix;
         const uint32_t peers = __match_any_sync(kFull, d);
         const int leader = __ffs(peers) - 1;
-        uint32_t before = 0;
-        if (lane == leader) before = atomicAdd(&sh_warp[wid][d], static_cast<uint32_t>(__popc(peers)));
+        const uint32_t before =
+            shared_add_if(&sh_warp[wid][d], static_cast<uint32_t>(__popc(peers)), lane == leader);
         const uint32_t r = __shfl_sync(kFull, before, leader) + __popc(peers & lt_mask);
         if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;  // two 16-bit ranks per register
     }
