@@ -136,6 +136,29 @@ def test_both_radix_pass_forms_give_the_same_bits(weighted, mean):
     assert_backward_matches(a, res, scale)
 
 
+def test_one_table_of_many_radix_tiles():
+    # ~4M lookups of one table: ~1000 radix tiles, so the slot scan cuts the
+    # table into dozens of segments; both pass forms and the oracle agree.
+    from paper_2609_30656_gb300.tbe import CB_SORT_LOOKBACK
+    g = torch.Generator().manual_seed(39)
+    rows, batch = 200000, 20000
+    table = (torch.randn(rows, 16, generator=g) * 0.01).float()
+    lens = torch.randint(0, 401, (batch,), generator=g)
+    off = torch.zeros(batch + 1, dtype=torch.int64)
+    off[1:] = torch.cumsum(lens, 0)
+    ind = torch.randint(0, rows, (int(off[-1]),), generator=g)
+    go = torch.randn(batch, 16, generator=g)
+    args = (ind.to(DEV), off.to(DEV), go.to(DEV))
+    a = _tbe([table]).backward(*args)
+    b = _tbe([table], extra_flags=CB_SORT_LOOKBACK).backward(*args)
+    torch.cuda.synchronize()
+    assert ind.numel() > 1000 * 4096 * 0.9
+    assert torch.equal(a.unique_ids[:a.num_unique], b.unique_ids[:b.num_unique])
+    assert torch.equal(a.grads[:a.num_floats], b.grads[:b.num_floats])
+    res, scale = backward_reference(np.array([rows]), np.array([16]), batch, ind, off, go, None, False)
+    assert_backward_matches(a, res, scale)
+
+
 def test_forced_lookback_timeout_returns_an_error_and_the_context_survives():
     from paper_2609_30656_gb300.tbe import CB_DEBUG_FORCE_LOOKBACK_TIMEOUT, CB_ERR_TIMEOUT
     # Enough lookups for several radix tiles; tile 1 waits on a word nothing writes.
