@@ -202,20 +202,41 @@ __global__ void __launch_bounds__(1024) rle_scan_kernel(const int64_t* tile_head
     if (threadIdx.x == 0) *num_unique = total;
 }
 
+// Each warp writes its run heads (unique key, start position) 32 at a time,
+// coalesced: lane l writes the warp's head x = x0 + l, found by a search over
+// the lanes' head prefixes (the owning lane) and then among that lane's 16 head
+// flags. With few repeats nearly every position is a head, and per-thread
+// stores would land 16 apart across the warp.
 __global__ void __launch_bounds__(kRleThreads) rle_write_kernel(const uint32_t* keys, int64_t n,
                                                                 const int64_t* tile_base,
                                                                 const int64_t* num_unique,
                                                                 uint32_t* uniq, uint32_t* seg_start) {
     __shared__ int64_t sh[33];
+    const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * kRleTile + threadIdx.x * kRleItems;
     const uint32_t flags = head_flags(keys, n, base);
     int64_t total;
-    int64_t u = tile_base[blockIdx.x] + block_excl_scan(__popc(flags), sh, &total);
-    for (uint32_t f = flags; f; f &= f - 1) {
-        const int i = __ffs(f) - 1;
-        uniq[u] = __ldg(keys + base + i);
-        seg_start[u] = static_cast<uint32_t>(base + i);
-        ++u;
+    const int64_t k = block_excl_scan(__popc(flags), sh, &total);
+    const int64_t wk = __shfl_sync(kFull, k, 0);                  // the warp's first head in the tile
+    const int32_t mine = static_cast<int32_t>(k - wk);            // this lane's first head in the warp
+    const int32_t wtot = __shfl_sync(kFull, mine + __popc(flags), 31);
+    uint32_t* uo = uniq + tile_base[blockIdx.x] + wk;
+    uint32_t* so = seg_start + tile_base[blockIdx.x] + wk;
+    const int64_t wbase = base - static_cast<int64_t>(lane) * kRleItems;  // lane 0's first position
+    for (int32_t x0 = 0; x0 < wtot; x0 += 32) {
+        const int32_t x = x0 + lane;
+        int j = 0;  // the last lane whose first head is at or before x: it holds head x
+#pragma unroll
+        for (int b = 16; b >= 1; b >>= 1)
+            if (__shfl_sync(kFull, mine, j + b) <= x) j += b;
+        uint32_t f = __shfl_sync(kFull, flags, j);
+        const int32_t mj = __shfl_sync(kFull, mine, j);
+        if (x < wtot) {
+            for (int32_t r = x - mj; r > 0; --r) f &= f - 1;  // drop the lane's earlier heads
+            const int64_t pos = wbase + static_cast<int64_t>(j) * kRleItems + (__ffs(f) - 1);
+            uo[x] = __ldg(keys + pos);
+            so[x] = static_cast<uint32_t>(pos);
+        }
     }
     if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) seg_start[*num_unique] = static_cast<uint32_t>(n);
 }
