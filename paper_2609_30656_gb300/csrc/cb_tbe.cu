@@ -58,6 +58,7 @@ struct Workspace {
     float* carry_head = nullptr;
     float* carry_tail = nullptr;
     int64_t* tail_owner = nullptr;
+    uint32_t* chunk_next = nullptr;
     int64_t max_chunks = 0;
     // radix sort plan: table-aligned tiles
     int64_t* sp_table_pos = nullptr;
@@ -155,6 +156,7 @@ size_t layout(const cb_tbe* h, int64_t B, int64_t n, char* base, Workspace* w) {
     ws.carry_head = static_cast<float*>(take(sizeof(float) * max_chunks * h->dmax));
     ws.carry_tail = static_cast<float*>(take(sizeof(float) * max_chunks * h->dmax));
     ws.tail_owner = static_cast<int64_t*>(take(sizeof(int64_t) * max_chunks));
+    ws.chunk_next = static_cast<uint32_t*>(take(sizeof(uint32_t) * (nc + 1)));
     for (int i = 0; i < 2; ++i) {
         ws.keys[i] = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
         ws.vals[i] = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
@@ -257,6 +259,7 @@ Plan make_plan(const cb_tbe* h, const Workspace& w, bool bwd, int64_t chunk_len)
     Q.carry_head = w.carry_head;
     Q.carry_tail = w.carry_tail;
     Q.tail_owner = w.tail_owner;
+    Q.chunk_next = w.chunk_next;
     return Q;
 }
 
@@ -354,6 +357,7 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     SQ.max_chunks = w.sp_max_tiles;
     SQ.carry_head = SQ.carry_tail = nullptr;
     SQ.tail_owner = nullptr;
+    SQ.chunk_next = nullptr;
     launch_plan(P, SQ, 2, nullptr, nullptr, h->num_sms, true, stream);
     h->launches += 2;
     if (lookback) {

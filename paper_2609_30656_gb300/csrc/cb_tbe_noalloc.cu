@@ -210,6 +210,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
         Q.carry_head = reinterpret_cast<float*>(base + o_hd);
         Q.carry_tail = reinterpret_cast<float*>(base + o_tl);
         Q.tail_owner = reinterpret_cast<int64_t*>(base + o_to);
+        Q.chunk_next = nullptr;
         launch_plan(P, Q, 0, nullptr, nullptr, num_sms, true, stream);
         for (size_t c = 0; c < classes.size(); ++c)
             launch_fwd_gather(P, Q, out, static_cast<int>(c), classes[c].dtype, classes[c].vpl,

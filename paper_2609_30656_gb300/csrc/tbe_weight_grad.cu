@@ -71,7 +71,8 @@ __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_
     const int g = lane / V, v = lane - g * V;
     const int64_t cb = Q.class_chunk_base[cls];
     const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
-    for (int64_t j = cb + warp_id_global(); j < ce; j += warps_in_grid()) {
+    for (int64_t j = first_chunk(Q, cls, cb, lane); j < ce;) {
+        const int64_t nxt = fetch_next_chunk(Q, cls, cb, j, lane);
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];
@@ -131,6 +132,7 @@ __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_
                 }
             }
         }
+        j = __shfl_sync(kFull, nxt, 0);
     }
 }
 
