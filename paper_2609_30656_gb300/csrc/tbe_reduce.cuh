@@ -13,6 +13,9 @@
 #ifndef CB_REDUCE_HALF_ROWS
 #define CB_REDUCE_HALF_ROWS 4  // rows in flight per lane for fp16 / bf16 grad_out
 #endif
+#ifndef CB_REDUCE_HALF_FAST_BATCH
+#define CB_REDUCE_HALF_FAST_BATCH 1  // fp16 / bf16 grad_out: unrolled path for batches with no run end
+#endif
 
 namespace cbtbe {
 
@@ -156,7 +159,7 @@ struct BwdPolicy {
     static constexpr int kUnroll = kRows / VPL > 0 ? kRows / VPL : 1;
     static constexpr bool kWeighted = PACKED;
     static constexpr bool kUnrollGroups = GO == CB_F32 ? CB_REDUCE_UNROLL_GROUPS : false;
-    static constexpr bool kFastBatch = GO == CB_F32 ? CB_REDUCE_FAST_BATCH : true;
+    static constexpr bool kFastBatch = GO == CB_F32 ? CB_REDUCE_FAST_BATCH : CB_REDUCE_HALF_FAST_BATCH;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;
