@@ -145,6 +145,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
     const size_t o_hd = off; off += up256(sizeof(float) * max_chunks * dmax);
     const size_t o_tl = off; off += up256(sizeof(float) * max_chunks * dmax);
     const size_t o_to = off; off += up256(sizeof(int64_t) * max_chunks);
+    const size_t o_nx = off; off += up256(sizeof(uint32_t) * (nc + 1));  // chunk counters
     if (off > kScratchBytes) return CB_ERR_CAPACITY;
 
     int device = -1;
@@ -210,7 +211,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
         Q.carry_head = reinterpret_cast<float*>(base + o_hd);
         Q.carry_tail = reinterpret_cast<float*>(base + o_tl);
         Q.tail_owner = reinterpret_cast<int64_t*>(base + o_to);
-        Q.chunk_next = nullptr;
+        Q.chunk_next = reinterpret_cast<uint32_t*>(base + o_nx);  // zeroed by the plan
         launch_plan(P, Q, 0, nullptr, nullptr, num_sms, true, stream);
         for (size_t c = 0; c < classes.size(); ++c)
             launch_fwd_gather(P, Q, out, static_cast<int>(c), classes[c].dtype, classes[c].vpl,
