@@ -89,7 +89,7 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
     const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     // all classes' chunks in one sequence: the counter after the classes' own
     for (int64_t j = first_chunk(Q, Q.num_classes, 0, lane); j < total;) {
-        const int64_t nxt = fetch_next_chunk(Q, Q.num_classes, 0, j, lane);
+        const int64_t nxt = fetch_next_chunk(Q, Q.num_classes, 0, lane);
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];

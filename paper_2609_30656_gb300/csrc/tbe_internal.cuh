@@ -121,8 +121,7 @@ struct Plan {
     float* carry_tail;                 // [max_chunks, dmax] piece of a segment begun here
     int64_t* tail_owner;               // [max_chunks] segment whose tail piece is here, or -1
     uint32_t* chunk_next;              // [num_classes + 1] next chunk to hand out per class, and
-                                       // over all classes (zeroed by the plan), or null: chunks
-                                       // round-robin over the warps
+                                       // over all classes (zeroed by the plan)
 };
 
 
@@ -143,16 +142,14 @@ __device__ __forceinline__ int64_t warps_in_grid() {
     return (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
 }
 
-// The walkers' chunk order: warps take the next chunk of their class from a
+// The walkers' chunk order: a warp takes the next chunk of its class from a
 // counter (lane 0 fetches the one after while the warp walks the current one),
-// or, without a counter, chunks round-robin. Either way chunks start in order.
+// so chunks start in order and cheap chunks do not leave warps idle.
 __device__ __forceinline__ int64_t first_chunk(const Plan& Q, int cls, int64_t cb, int lane) {
-    if (!Q.chunk_next) return cb + warp_id_global();
     const int64_t j = lane == 0 ? cb + atomicAdd(Q.chunk_next + cls, 1u) : 0;
     return __shfl_sync(kFull, j, 0);
 }
-__device__ __forceinline__ int64_t fetch_next_chunk(const Plan& Q, int cls, int64_t cb, int64_t j, int lane) {
-    if (!Q.chunk_next) return j + warps_in_grid();
+__device__ __forceinline__ int64_t fetch_next_chunk(const Plan& Q, int cls, int64_t cb, int lane) {
     return lane == 0 ? cb + atomicAdd(Q.chunk_next + cls, 1u) : 0;
 }
 

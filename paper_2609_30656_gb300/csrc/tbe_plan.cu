@@ -120,7 +120,7 @@ __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* 
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     const int64_t C = Q.chunk_len;
     const int64_t U = mode == 1 ? *num_unique : 0;
-    if (blockIdx.x == 0 && Q.chunk_next)
+    if (blockIdx.x == 0 && Q.chunk_next)  // the walkers' chunk counters (none for sort tiles)
         for (int c = threadIdx.x; c <= Q.num_classes; c += blockDim.x) Q.chunk_next[c] = 0;
     for (int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; j < total;
          j += stride) {

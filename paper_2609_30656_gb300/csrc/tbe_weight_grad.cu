@@ -72,7 +72,7 @@ __global__ void __launch_bounds__(kWarpThreads) weight_grad_kernel(const __grid_
     const int64_t cb = Q.class_chunk_base[cls];
     const int64_t ce = min64(Q.class_chunk_base[cls + 1], Q.max_chunks);
     for (int64_t j = first_chunk(Q, cls, cb, lane); j < ce;) {
-        const int64_t nxt = fetch_next_chunk(Q, cls, cb, j, lane);
+        const int64_t nxt = fetch_next_chunk(Q, cls, cb, lane);
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];
