@@ -237,7 +237,10 @@ cb_status cb_tbe_backward_apply(cb_tbe* h, int32_t batch, const void* indices, i
  *   kind, lr, eps, state: as in cb_tbe_backward_apply
  * THIS CALL WRITES THE TABLES given to cb_tbe_create (and the state arrays).
  * Errors: CB_ERR_INVALID_ARG for a NULL or misaligned buffer, an unknown kind,
- * a NaN lr, eps < 0 or a missing state; CB_ERR_CUDA if the launch fails. */
+ * a NaN lr, eps < 0 or a missing state; CB_ERR_CUDA if the launch fails; a row
+ * whose id or offset does not fit this handle's tables or g's F (buffers not
+ * written by this handle) is skipped and sets CB_ERR_INDEX_OOB (sticky; returned
+ * now under CB_VALIDATE, else by cb_tbe_get_error). */
 cb_status cb_tbe_apply_sparse(cb_tbe* h, const cb_sparse_grad* g, cb_optimizer kind, float lr, float eps,
                               float* const* state, cudaStream_t stream);
 

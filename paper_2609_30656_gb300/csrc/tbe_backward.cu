@@ -487,7 +487,8 @@ __global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid
     static_assert(32 % R == 0, "rows per step divide the warp's 32");
     const int lane = threadIdx.x & 31;
     const int64_t U = *O.num_unique;
-    if (U > O.cap_rows || *O.num_floats > O.cap_floats) return;
+    const int64_t F = *O.num_floats;
+    if (U > O.cap_rows || F > O.cap_floats) return;
     const bool adagrad = O.apply == kApplyAdagrad;
     for (int64_t u0 = warp_id_global() * 32; u0 < U; u0 += warps_in_grid() * 32) {
         // this lane's row: start of its stored row, of its gradient and state
@@ -502,12 +503,17 @@ __global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid
         }
         const TableDev& td = P.tables[lo];
         const int64_t row = id - td.row_base;
-        const unsigned long long my_row = reinterpret_cast<unsigned long long>(row_ptr(td, row));
-        const unsigned long long my_grad = reinterpret_cast<unsigned long long>(O.grads + goff);
+        // A gradient this handle's backward wrote always passes; a row that
+        // does not (buffers from elsewhere) is skipped and reported, never
+        // followed outside a table, the gradient or the state.
+        const bool ok = row >= 0 && row < td.rows && goff >= 0 && goff + td.dim <= F;
+        if (!ok && u0 + lane < U) set_error(P.error, CB_ERR_INDEX_OOB);
+        const unsigned long long my_row = reinterpret_cast<unsigned long long>(row_ptr(td, ok ? row : 0));
+        const unsigned long long my_grad = reinterpret_cast<unsigned long long>(O.grads + (ok ? goff : 0));
         const unsigned long long my_state =
-            adagrad ? reinterpret_cast<unsigned long long>(O.state[lo] + row) : 0ull;
-        const int my_shape = (td.dim << 2) | td.dtype;
-        const float my_m0 = adagrad ? *reinterpret_cast<const float*>(my_state) : 0.f;
+            adagrad && ok ? reinterpret_cast<unsigned long long>(O.state[lo] + row) : 0ull;
+        const int my_shape = ((ok ? td.dim : 0) << 2) | td.dtype;  // dim 0: nothing loaded or stored
+        const float my_m0 = my_state ? *reinterpret_cast<const float*>(my_state) : 0.f;
         const int rows_here = static_cast<int>(min64(32, U - u0));
         for (int r0 = 0; r0 < rows_here; r0 += R) {
             char* rp[R];
@@ -552,7 +558,7 @@ __global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid
                 for (int i = 0; i < R; ++i)
                     if (lane == r0 + i) mine = sq[i];
                 float my_scale = O.lr;
-                if (lane >= r0 && lane < r0 + R && lane < rows_here) {
+                if (lane >= r0 && lane < r0 + R && lane < rows_here && my_state) {
                     const float m = my_m0 + mine / static_cast<float>(my_shape >> 2);
                     *reinterpret_cast<float*>(my_state) = m;
                     my_scale = O.lr / (sqrtf(m) + O.eps);

@@ -237,3 +237,29 @@ def test_cfg2_full_size_two_pass_equals_fused():
         assert torch.equal(x, y)
     for x, y in zip(sa, sc):
         np.testing.assert_array_equal(x, y)
+
+
+def test_two_pass_skips_rows_that_are_not_this_handles():
+    # A gradient written by a handle over a 1000-row table, applied through a
+    # handle over a 10-row table: ids >= 10 are skipped and reported, ids < 10
+    # are stepped as usual; nothing outside the small table is touched.
+    from paper_2609_30656_gb300.tbe import CB_ERR_INDEX_OOB, TBE
+    g_ = torch.Generator().manual_seed(19)
+    big = (torch.randn(1000, 16, generator=g_) * 0.01).to(DEV)
+    small_host = (torch.randn(10, 16, generator=g_) * 0.01)
+    small = small_host.to(DEV)
+    off = torch.tensor([0, 3, 7, 12], dtype=torch.int64)
+    ind = torch.tensor([1, 5, 900, 2, 2, 999, 7, 10, 3, 4, 500, 9], dtype=torch.int64)
+    go = torch.randn(3, 16, generator=g_)
+    m_big, m_small = TBE([big]), TBE([small])
+    g = m_big.backward(ind.to(DEV), off.to(DEV), go.to(DEV))
+    m_small.apply_sparse(g, optimizer="sgd", lr=1.0)
+    assert m_small.get_error() == CB_ERR_INDEX_OOB
+    ids = g.unique_ids[:g.num_unique].cpu()
+    offs = g.grad_offsets[:g.num_unique].cpu()
+    grads = g.grads[:g.num_floats].cpu()
+    want = small_host.clone()
+    for k, r in enumerate(ids.tolist()):
+        if r < 10:
+            want[r] -= grads[int(offs[k]):int(offs[k]) + 16]
+    assert torch.equal(small.cpu(), want)
