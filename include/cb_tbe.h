@@ -33,7 +33,10 @@
  *     Device-side checks (index range; offsets under CB_VALIDATE) never trap:
  *     they set a sticky error word. Under CB_VALIDATE the call synchronises
  *     `stream` and returns that error; otherwise cb_tbe_get_error() returns
- *     it later. An out-of-range index contributes nothing to the output.
+ *     it later. An out-of-range index (negative, or >= rows_t) contributes
+ *     nothing: not to the pooled output, not to any gradient row (its row is not
+ *     listed unless a valid lookup touches it) and not to any optimizer step.
+ *     For mean pooling the bag length L still counts it, as in the forward.
  *   - Results are deterministic: the same inputs give bit-identical outputs.
  */
 #ifndef CB_TBE_H
@@ -97,7 +100,8 @@ typedef struct cb_tbe cb_tbe;
 /* Creates a handle on the current CUDA device for `num_tables` tables (the
  * descriptors are copied; the table memory stays the caller's). `mode` picks
  * sum or mean pooling; `idx_dtype` is the type of both indices and offsets.
- * The sum of all rows must be below 2^32 and num_tables * batch below 2^31.
+ * The sum of all rows plus num_tables must be below 2^32 (the backward's sort
+ * keys: each table's rows and one spare key) and num_tables * batch below 2^31.
  * Returns CB_ERR_INVALID_ARG for a bad descriptor, CB_ERR_CUDA / CB_ERR_OOM
  * if the device set-up fails. On success *out receives the handle. */
 cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pooling mode,
@@ -134,12 +138,13 @@ cb_status cb_tbe_forward(cb_tbe* h, int32_t batch, const void* indices, int64_t 
  * table (e.g. up to ~7.9 M lookups over 100 tables of dim 128); a larger call
  * is refused with CB_ERR_CAPACITY before any GPU work.
  * The first call on each device looks up the array's device address (with
- * that device current); make that first call before any stream capture.
- * Every call reuses the same array (its error word is cleared at the start of
- * each call), so calls whose GPU work overlaps race: do not run two at once
- * from several threads or streams. The call checks the offsets, synchronises
- * `stream` and returns the device-side status (as under CB_VALIDATE). It calls
- * no cudaMalloc, cudaFree or allocating library routine. */
+ * that device current). Every call reuses the same array (its error word is
+ * cleared at the start of each call), so calls whose GPU work overlaps race:
+ * do not run two at once from several threads or streams. The call checks the
+ * offsets, then synchronises `stream` and reads the device-side status back
+ * (as under CB_VALIDATE), which is why it cannot be called while `stream` is
+ * being captured into a CUDA graph. It calls no cudaMalloc, cudaFree or
+ * allocating library routine. */
 cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t num_tables, cb_pooling mode,
                                  cb_index_dtype idx_dtype, int32_t batch, const void* indices,
                                  int64_t num_indices, const void* offsets,
@@ -190,6 +195,19 @@ const char* cb_tbe_component_name(int32_t i);
 
 /* Number of CUDA kernels this handle has launched since creation. */
 uint64_t cb_tbe_launch_count(const cb_tbe* h);
+
+/* Test and debugging aid (not in the paper): the order the backward's stable
+ * radix sort produced. Copies, on `stream`, the sorted payloads of the last
+ * cb_tbe_backward or cb_tbe_backward_apply call on this handle into the device
+ * array out[num_indices]: entry k belongs to the lookup at sorted position k
+ * (each table's lookups by ascending row, ties in lookup order, lookups with an
+ * out-of-range index after the table's rows). The payload is the lookup's
+ * position in `indices` when that call had per-sample weights or mean pooling,
+ * and otherwise its bag t*B + b (0xffffffff for an out-of-range index).
+ * num_indices must equal that call's; the payloads stay in the handle's
+ * workspace until its next backward call or until the workspace grows.
+ * CB_ERR_INVALID_ARG when no such payloads are held. */
+cb_status cb_tbe_sorted_payloads(const cb_tbe* h, uint32_t* out, int64_t num_indices, cudaStream_t stream);
 
 /* Short English description of a status code. */
 const char* cb_tbe_status_string(cb_status s);

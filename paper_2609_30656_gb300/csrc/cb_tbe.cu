@@ -82,8 +82,11 @@ struct Workspace {
     uint32_t* uniq = nullptr;
     uint32_t* seg_start = nullptr;
     int64_t* table_first = nullptr;
+    int64_t* live_end = nullptr;
+    int64_t* out_first = nullptr;
     int64_t* float_base = nullptr;
     int64_t* num_unique = nullptr;
+    int64_t* out_sizes = nullptr;  // [2] U and F of a fused step (no caller buffers)
     int* cap_fail = nullptr;
     int4* heavy = nullptr;
     uint32_t* heavy_count = nullptr;
@@ -125,6 +128,9 @@ struct cb_tbe {
     void* ws = nullptr;
     size_t ws_bytes = 0;
     cudaStream_t last_stream = nullptr;
+    // Sorted payloads of the last backward that reached the sort (workspace).
+    const uint32_t* last_sorted = nullptr;
+    int64_t last_sorted_n = 0;
     cudaEvent_t ev_fwd[4] = {};
     cudaEvent_t ev_bwd[5] = {};
     bool fwd_timed = false;
@@ -189,8 +195,11 @@ size_t layout(const cb_tbe* h, int64_t B, int64_t n, char* base, Workspace* w) {
     ws.uniq = static_cast<uint32_t*>(take(sizeof(uint32_t) * n));
     ws.seg_start = static_cast<uint32_t*>(take(sizeof(uint32_t) * (n + 1)));
     ws.table_first = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
+    ws.live_end = static_cast<int64_t*>(take(sizeof(int64_t) * T));
+    ws.out_first = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
     ws.float_base = static_cast<int64_t*>(take(sizeof(int64_t) * (T + 1)));
     ws.num_unique = static_cast<int64_t*>(take(sizeof(int64_t)));
+    ws.out_sizes = static_cast<int64_t*>(take(sizeof(int64_t) * 2));
     ws.cap_fail = static_cast<int*>(take(sizeof(int)));
     ws.max_heavy = max_chunks / 32 + 1;  // a heavy run owns more than 32 chunks
     ws.heavy = static_cast<int4*>(take(sizeof(int4) * ws.max_heavy));
@@ -207,6 +216,7 @@ cb_status ensure_workspace(cb_tbe* h, int64_t B, int64_t n) {
         cudaFree(h->ws);
         h->ws = nullptr;
         h->ws_bytes = 0;
+        h->last_sorted = nullptr;
     }
     if (cudaMalloc(&h->ws, need) != cudaSuccess) {
         cudaGetLastError();
@@ -307,6 +317,7 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
     h->last_stream = stream;
     h->bwd_timed = false;
+    h->last_sorted = nullptr;
     Problem P = make_problem(h, batch, indices, n, offsets, per_sample_weights);
     record(h, h->ev_bwd[0], stream);
     if ((h->flags & CB_VALIDATE) && batch > 0) {
@@ -402,6 +413,8 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
         cur ^= 1;
     }
     record(h, h->ev_bwd[2], stream);
+    h->last_sorted = w.vals[cur];
+    h->last_sorted_n = n;
 
     // (3) runs of equal ids, (4) per-table ranges and capacity check
     launch_rle(w.keys[cur], n, w.tile_heads, w.tile_base, w.num_unique, w.uniq, w.seg_start, stream);
@@ -413,6 +426,8 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     O.uniq = w.uniq;
     O.num_unique_ws = w.num_unique;
     O.table_first = w.table_first;
+    O.live_end = w.live_end;
+    O.out_first = w.out_first;
     O.float_base = w.float_base;
     O.cap_fail = w.cap_fail;
     O.heavy = w.heavy;
@@ -421,12 +436,12 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
     if (a) {
         // No caller buffers: the sizes land in the workspace's own words.
         O.unique_ids = nullptr;
-        O.table_offsets = w.table_first;
+        O.table_offsets = nullptr;
         O.grad_offsets = nullptr;
         O.grads = nullptr;
         O.cap_rows = O.cap_floats = INT64_MAX;
-        O.num_unique = w.num_unique;
-        O.num_floats = w.float_base + h->T;
+        O.num_unique = w.out_sizes;
+        O.num_floats = w.out_sizes + 1;
         O.apply = a->kind;
         O.lr = a->lr;
         O.eps = a->eps;
@@ -529,6 +544,7 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
         td.data = d.data;
         td.rows = d.rows;
         td.row_base = row_base;
+        td.key_base = row_base + t;  // one spare key per table: out-of-range lookups
         td.dim = d.dim;
         td.doff = static_cast<int32_t>(doff);
         td.dtype = d.dtype;
@@ -541,17 +557,19 @@ cb_status cb_tbe_create(const cb_table_desc* tables, int32_t num_tables, cb_pool
         h->dmax = std::max(h->dmax, d.dim);
         h->tables.push_back(td);
     }
-    if (row_base >= (int64_t(1) << 32) || doff >= (int64_t(1) << 31) || h->dmax > 512) {
+    // Backward keys: every table's rows plus one spare key, all below 2^32.
+    if (row_base + num_tables >= (int64_t(1) << 32) || doff >= (int64_t(1) << 31) || h->dmax > 512) {
         delete h;
         return CB_ERR_INVALID_ARG;
     }
     h->sum_rows = row_base;
     h->sum_d = static_cast<int32_t>(doff);
-    // Each table's range is sorted on its own, on the bits of the row number.
+    // Each table's range is sorted on its own, on the bits of the row number
+    // r <= rows_t (r = rows_t: an out-of-range lookup).
     int64_t max_rows = 1;
     for (const TableDev& td : h->tables) max_rows = std::max(max_rows, td.rows);
     int bits = 1;
-    while (bits < 32 && (int64_t(1) << bits) < max_rows) ++bits;
+    while (bits < 32 && (int64_t(1) << bits) <= max_rows) ++bits;
     h->key_bits = bits;
     h->passes = (bits + 7) / 8;
 
@@ -819,6 +837,17 @@ cb_status cb_tbe_last_timings(cb_tbe* h, float* ms, int32_t n) {
 }
 
 uint64_t cb_tbe_launch_count(const cb_tbe* h) { return h ? h->launches : 0; }
+
+cb_status cb_tbe_sorted_payloads(const cb_tbe* h, uint32_t* out, int64_t num_indices, cudaStream_t stream) {
+    if (!h || !out || !h->last_sorted || num_indices != h->last_sorted_n) return CB_ERR_INVALID_ARG;
+    if (!current_device_ok(h)) return CB_ERR_INVALID_ARG;
+    if (cudaMemcpyAsync(out, h->last_sorted, sizeof(uint32_t) * num_indices, cudaMemcpyDeviceToDevice,
+                        stream) != cudaSuccess) {
+        cudaGetLastError();
+        return CB_ERR_CUDA;
+    }
+    return CB_OK;
+}
 
 void cb_tbe_destroy(cb_tbe* h) {
     if (!h) return;

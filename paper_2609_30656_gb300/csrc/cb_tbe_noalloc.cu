@@ -99,6 +99,7 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
         x.data = d.data;
         x.rows = d.rows;
         x.row_base = row_base;
+        x.key_base = row_base + t;
         x.dim = d.dim;
         x.doff = static_cast<int32_t>(doff);
         x.dtype = d.dtype;
@@ -132,6 +133,11 @@ extern "C" cb_status cb_tbe_forward_noalloc(const cb_table_desc* tables, int32_t
     // Layout of the static scratch for this call; refuse calls that do not fit.
     const int64_t T = num_tables, nc = static_cast<int64_t>(classes.size());
     const int64_t max_chunks = num_indices / kChunk + T + 1;
+    // Each chunk takes a descriptor, an owner word and two carry rows; refuse a
+    // call whose chunks alone exceed the array before any product below can
+    // wrap around (num_indices near 2^63).
+    const size_t per_chunk = sizeof(Chunk) + sizeof(int64_t) + 2 * sizeof(float) * static_cast<size_t>(dmax);
+    if (max_chunks > static_cast<int64_t>(kScratchBytes / per_chunk)) return CB_ERR_CAPACITY;
     size_t off = 0;
     const size_t o_err = off; off += up256(sizeof(int));
     const size_t o_zero = off; off += up256(2048);

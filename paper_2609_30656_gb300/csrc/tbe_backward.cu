@@ -3,7 +3,7 @@
 //   G[row_base_t + r] = sum_{i : table t, indices[i] == r} w_i * s_b(i) * grad_out[b(i), Doff_t ..]
 //
 // Steps: (1) key generation: one warp per chunk of lookups walks the bags and
-// writes key_i = row_base_t + indices[i] with a payload (the bag id, or the
+// writes key_i = key_base_t + indices[i] with a payload (the bag id, or the
 // lookup position plus a packed (bag, w_i * s_b) pair when a coefficient is
 // needed); (2) radix sort of each table's range;
 // (3) run-length pass over the sorted ids; (4) per-table unique ranges and
@@ -93,7 +93,7 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
         const Chunk ch = Q.chunks[j];
         const int t = ch.table;
         const TableDev& td = P.tables[t];
-        const int64_t rows = td.rows, row_base = td.row_base;
+        const int64_t rows = td.rows, key_base = td.key_base;
         const int64_t k0 = ch.k0;
         const int32_t len = static_cast<int32_t>(ch.len & 0x7fffffffu);
         const int64_t bag_lo = static_cast<int64_t>(t) * P.B, bag_hi = bag_lo + P.B;
@@ -122,19 +122,24 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
                     set_error(P.error, CB_ERR_BAD_OFFSETS);
                     my_bag = bag_hi - 1;
                 }
+                // An out-of-range index takes the table's spare key (it sorts
+                // after every row into a run the reduce drops) and a bag outside
+                // the table: it contributes to no gradient row.
                 int64_t r = idx[u];
+                uint32_t bag = static_cast<uint32_t>(my_bag);
                 if (r < 0 || r >= rows) {
                     set_error(P.error, CB_ERR_INDEX_OOB);
-                    r = r < 0 ? 0 : rows - 1;
+                    r = rows;
+                    bag = kDeadBag;
                 }
-                keys[q] = static_cast<uint32_t>(row_base + r);
+                keys[q] = static_cast<uint32_t>(key_base + r);
                 if (PACKED) {
                     float c = wt[u];
                     if (P.mean && my_e > my_s) c = c / static_cast<float>(my_e - my_s);
                     vals[q] = static_cast<uint32_t>(k0 + q);
-                    K.packed[k0 + q] = make_uint2(static_cast<uint32_t>(my_bag), __float_as_uint(c));
+                    K.packed[k0 + q] = make_uint2(bag, __float_as_uint(c));
                 } else {
-                    vals[q] = static_cast<uint32_t>(my_bag);
+                    vals[q] = bag;
                 }
             }
         }
@@ -248,45 +253,65 @@ __global__ void __launch_bounds__(kRleThreads) rle_write_kernel(const uint32_t* 
 
 __global__ void __launch_bounds__(1024) bwd_finalize_kernel(Problem P, BwdOut O) {
     __shared__ int64_t sh[33];
-    __shared__ int64_t running;
+    __shared__ int64_t run_rows, run_floats;
     const int64_t U = *O.num_unique_ws;
+    // First run of each table: the first run key at or above key_base_t.
     for (int t = threadIdx.x; t <= P.T; t += blockDim.x) {
-        const int64_t rb = t < P.T ? P.tables[t].row_base
-                                   : P.tables[P.T - 1].row_base + P.tables[P.T - 1].rows;
+        const int64_t kb = t < P.T ? P.tables[t].key_base
+                                   : P.tables[P.T - 1].key_base + P.tables[P.T - 1].rows + 1;
         int64_t a = 0, b = U;
         while (a < b) {
             const int64_t m = (a + b) >> 1;
-            if (static_cast<int64_t>(O.uniq[m]) < rb) a = m + 1; else b = m;
+            if (static_cast<int64_t>(O.uniq[m]) < kb) a = m + 1; else b = m;
         }
         O.table_first[t] = a;
     }
-    if (threadIdx.x == 0) running = 0;
+    if (threadIdx.x == 0) run_rows = run_floats = 0;
     __syncthreads();
+    // A table's last run may hold its out-of-range lookups (the spare key):
+    // it is not output. Output rows and floats are scanned over the rest.
     for (int t0 = 0; t0 < P.T; t0 += blockDim.x) {
         const int t = t0 + threadIdx.x;
-        const int64_t c = t < P.T ? (O.table_first[t + 1] - O.table_first[t]) * P.tables[t].dim : 0;
-        int64_t total;
-        const int64_t ex = block_excl_scan(c, sh, &total);
-        if (t < P.T) O.float_base[t] = running + ex;
+        int64_t live = 0, dim = 0;
+        if (t < P.T) {
+            const TableDev& td = P.tables[t];
+            const int64_t a = O.table_first[t], b = O.table_first[t + 1];
+            const bool dead = b > a && static_cast<int64_t>(O.uniq[b - 1]) == td.key_base + td.rows;
+            O.live_end[t] = dead ? b - 1 : b;
+            live = (dead ? b - 1 : b) - a;
+            dim = td.dim;
+        }
+        int64_t rows_total, floats_total;
+        const int64_t ex_rows = block_excl_scan(live, sh, &rows_total);
+        const int64_t ex_floats = block_excl_scan(live * dim, sh, &floats_total);
+        if (t < P.T) {
+            O.out_first[t] = run_rows + ex_rows;
+            O.float_base[t] = run_floats + ex_floats;
+        }
         __syncthreads();
-        if (threadIdx.x == 0) running += total;
+        if (threadIdx.x == 0) {
+            run_rows += rows_total;
+            run_floats += floats_total;
+        }
         __syncthreads();
     }
-    const int64_t F = running;
-    for (int t = threadIdx.x; t <= P.T; t += blockDim.x) O.table_offsets[t] = O.table_first[t];
+    const int64_t Uo = run_rows, F = run_floats;
+    if (O.table_offsets)
+        for (int t = threadIdx.x; t <= P.T; t += blockDim.x) O.table_offsets[t] = t < P.T ? O.out_first[t] : Uo;
     if (threadIdx.x == 0) {
+        O.out_first[P.T] = Uo;
         O.float_base[P.T] = F;
-        *O.num_unique = U;
+        *O.num_unique = Uo;
         *O.num_floats = F;
         int fail = 0;
         // After a timed-out sort pass the sorted order is not trustworthy.
         if (*reinterpret_cast<volatile int*>(P.error) == CB_ERR_TIMEOUT) fail = 1;
-        if (O.grads && (U > O.cap_rows || F > O.cap_floats)) {
+        if (O.grads && (Uo > O.cap_rows || F > O.cap_floats)) {
             set_error(P.error, CB_ERR_CAPACITY);
             fail = 1;
         }
         *O.cap_fail = fail;
-        if (O.grads && !fail) O.grad_offsets[U] = F;
+        if (O.grads && !fail) O.grad_offsets[Uo] = F;
     }
 }
 
@@ -394,7 +419,7 @@ __global__ void __launch_bounds__(kWarpThreads) bwd_apply_split_kernel(const __g
             const int64_t seg = __shfl_sync(kFull, mine, b);
             const int t = Q.chunks[j].table;
             const TableDev& td = P.tables[t];
-            const int64_t row = static_cast<int64_t>(O.uniq[seg]) - td.row_base;
+            const int64_t row = static_cast<int64_t>(O.uniq[seg]) - td.key_base;
             const float* g = Q.carry_tail + j * P.dmax;
             float sq = 0.f;
             for (int x0 = lane * 4; x0 < td.dim; x0 += 128) {

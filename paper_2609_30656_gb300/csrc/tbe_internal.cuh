@@ -69,6 +69,11 @@ struct TableDev {
     const void* data;   // row-major [rows, dim] of dtype
     int64_t rows;
     int64_t row_base;   // rows of all tables before this one (global row id base)
+    // Backward sort key of row r: key_base + r, with key_base = row_base + t.
+    // Each table owns rows + 1 keys; key_base + rows marks a lookup whose index
+    // is out of range, which sorts after the table's rows into a run of its own
+    // that the reduce drops.
+    int64_t key_base;
     int32_t dim;
     int32_t doff;       // column offset of this table in the [B, sum dims] output
     int32_t dtype;      // cb_dtype

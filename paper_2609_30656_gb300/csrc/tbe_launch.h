@@ -10,7 +10,7 @@ struct Problem;
 struct Plan;
 
 // One radix pass over n (key, payload) pairs, each table's range sorted on
-// its own: tiles never straddle tables, digits are taken from key - row_base_t.
+// its own: tiles never straddle tables, digits are taken from key - key_base_t.
 struct SortPass {
     const uint32_t* keys_in;
     const uint32_t* vals_in;
@@ -21,7 +21,7 @@ struct SortPass {
     const int64_t* table_first_tile;  // [T + 1]
     const struct TableDev* tables;
     int64_t n;
-    int shift;                   // digit = ((key - row_base_t) >> shift) & 255
+    int shift;                   // digit = ((key - key_base_t) >> shift) & 255
     // reduce-then-scan
     const int64_t* table_pos;    // [T + 1] first position of each table
     uint32_t* tile_digits;       // [tiles][256]: digit counts, then first output slots
@@ -39,10 +39,15 @@ struct SortPass {
     uint64_t timeout_ns;
 };
 
+// Payload bag of a lookup whose index is out of range: outside every table's
+// bags, so the reduce reads the zero row for it.
+constexpr uint32_t kDeadBag = 0xffffffffu;
+
 struct KeyGen {
-    uint32_t* keys;    // [n] row_base_t + index
-    uint32_t* vals;    // [n] bag id, or lookup position when `packed` is used
-    uint2* packed;     // [n] (bag id, bits of w_i * s_b) by lookup position, or null
+    uint32_t* keys;    // [n] key_base_t + index (key_base_t + rows_t: out of range)
+    uint32_t* vals;    // [n] bag id (kDeadBag when out of range), or lookup position
+                       // when `packed` is used
+    uint2* packed;     // [n] (bag id or kDeadBag, bits of w_i * s_b) by lookup position, or null
 };
 
 struct BwdOut {
@@ -50,9 +55,13 @@ struct BwdOut {
     const uint32_t* seg_start;   // [U + 1]
     const uint32_t* vals_sorted; // [n]
     const uint2* packed;         // [n] or null
-    const uint32_t* uniq;        // [U]
-    int64_t* num_unique_ws;
-    int64_t* table_first;        // [T + 1]
+    const uint32_t* uniq;        // [U] sorted keys of the runs (key_base_t + r)
+    int64_t* num_unique_ws;      // U, runs of out-of-range lookups included
+    int64_t* table_first;        // [T + 1] first run of each table
+    int64_t* live_end;           // [T] one past table t's last run of real rows
+                                 // (table_first[t + 1], less the out-of-range run)
+    int64_t* out_first;          // [T + 1] first output row of each table (runs of
+                                 // out-of-range lookups are not output)
     int64_t* float_base;         // [T + 1]
     int* cap_fail;
     int4* heavy;                 // [max_heavy] runs left for the block-wide combine

@@ -129,7 +129,7 @@ template <int N>
 __device__ __noinline__ void apply_row(const Problem& P, const BwdOut& O, int t, int32_t seg,
                                        const GradRow<N> g, bool group0) {
     const TableDev& td = P.tables[t];
-    const int64_t row = static_cast<int64_t>(__ldg(O.uniq + seg)) - td.row_base;
+    const int64_t row = static_cast<int64_t>(__ldg(O.uniq + seg)) - td.key_base;
     float sq = 0.f;
 #pragma unroll
     for (int k = 0; k < N; ++k)
@@ -169,7 +169,9 @@ struct BwdPolicy {
     uint32_t stride;    // 16-byte vectors per grad_out row
     int32_t chunk;
     int32_t bag_lo;
-    int32_t seg_lo;     // first unique index of this table
+    int32_t seg_lo;     // first run of this table
+    int32_t out_shift;  // run index - output row (runs of out-of-range lookups of
+                        // earlier tables are not output)
     int32_t dim;
     int32_t table;
 
@@ -200,11 +202,12 @@ struct BwdPolicy {
         a = (b >= 0 && b < P.B) ? static_cast<uint32_t>(b) : kInvalid;
     }
     static constexpr bool kEmptySegments = false;
-    // Row id and float offset of a run that begins in this chunk.
+    // Row id (row_base_t + r = key - t) and float offset of a run that begins
+    // in this chunk, at its output row.
     __device__ __forceinline__ void seg_meta(int32_t seg) const {
         if (APPLY) return;  // a fused step writes no gradient buffers
-        O.unique_ids[seg] = __ldg(O.uniq + seg);
-        O.grad_offsets[seg] = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
+        O.unique_ids[seg - out_shift] = static_cast<int64_t>(__ldg(O.uniq + seg)) - table;
+        O.grad_offsets[seg - out_shift] = float_lo + static_cast<int64_t>(seg - seg_lo) * dim;
     }
     __device__ __forceinline__ void put_empty(int32_t, int, bool) const {}
     __device__ __forceinline__ void emit(int32_t seg, int32_t L, bool started, bool ends,
@@ -273,13 +276,16 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
         pol.chunk = static_cast<int32_t>(j);
         pol.bag_lo = t * P.B;
         pol.seg_lo = static_cast<int32_t>(O.table_first[t]);
+        pol.out_shift = static_cast<int32_t>(O.table_first[t] - O.out_first[t]);
         pol.dim = td.dim;
         pol.table = t;
         ChunkCtx c;
         c.k0 = ch.k0;
         c.len = static_cast<int32_t>(ch.len & 0x7fffffffu);
         c.first = static_cast<int32_t>(max64(ch.first, O.table_first[t]));
-        c.seg_hi = static_cast<int32_t>(O.table_first[t + 1]);
+        // The run of out-of-range lookups (the table's spare key, last) is
+        // walked but never output: its items read the zero row.
+        c.seg_hi = static_cast<int32_t>(O.live_end[t]);
         c.lanes = td.grad_lanes;
         c.groups = td.grad_groups;
         c.row_vecs = td.grad_vecs;

@@ -1,9 +1,10 @@
 // tbe_sort.cu -- stable LSD radix sort of (row id, payload) pairs for the
 // de-duplicated backward of the pooled embedding bag.
 //
-// A table's lookups are contiguous and its row ids are row_base_t + r with
-// r < rows_t, so each table's range is sorted on its own, on the bits of r only
-// (3 passes of 8 bits for tables of up to 16M rows), in tiles of at most 4096
+// A table's lookups are contiguous and its sort keys are key_base_t + r with
+// r <= rows_t (r = rows_t: an out-of-range index), so each table's range is
+// sorted on its own, on the bits of r only (3 passes of 8 bits for tables of
+// fewer than 16M rows), in tiles of at most 4096
 // positions that never straddle tables. A block ranks its tile's keys by digit
 // (warp match + per-warp counters, stable by position), lays them out by digit
 // in shared memory and writes each digit's run to that digit's slots of the
@@ -48,8 +49,8 @@ __device__ __forceinline__ void store_volatile(uint32_t* p, uint32_t v) {
 
 constexpr int kLookbackWindow = 8;  // predecessor tiles inspected per look-back round
 
-__device__ __forceinline__ uint32_t sort_digit(uint32_t key, uint32_t row_base, int shift) {
-    return ((key - row_base) >> shift) & (kRadix - 1);
+__device__ __forceinline__ uint32_t sort_digit(uint32_t key, uint32_t key_base, int shift) {
+    return ((key - key_base) >> shift) & (kRadix - 1);
 }
 
 // *p += v in the lanes where `on`, returning the old value there (0 elsewhere):
@@ -71,7 +72,7 @@ __device__ __forceinline__ uint32_t shared_add_if(uint32_t* p, uint32_t v, bool 
 // atomics take effect in issue order, so item j's lanes count before item
 // j + 1's, and lanes of one item by lane: the rank follows the position.
 // Positions past the tile count under the extra digit kRadix.
-__device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int tile_count, uint32_t row_base,
+__device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int tile_count, uint32_t key_base,
                                           int shift, uint32_t (*sh_warp)[kRadix + 1],
                                           uint32_t (&rank2)[kSortItems / 2]) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -79,7 +80,7 @@ __device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
-        const uint32_t d = local < tile_count ? sort_digit(key[j], row_base, shift) : kRadix;
+        const uint32_t d = local < tile_count ? sort_digit(key[j], key_base, shift) : kRadix;
         const uint32_t peers = __match_any_sync(kFull, d);
         const int leader = __ffs(peers) - 1;
         const uint32_t before =
@@ -93,13 +94,13 @@ __device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int
 // start + the warp's prefix + the rank): every slot first (the counters are
 // read-only here), then the stores.
 __device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], const uint32_t (&val)[kSortItems],
-                                             uint32_t (&rank2)[kSortItems / 2], int tile_count, uint32_t row_base,
+                                             uint32_t (&rank2)[kSortItems / 2], int tile_count, uint32_t key_base,
                                              int shift, const uint32_t (*sh_warp)[kRadix + 1],
                                              const uint32_t* sh_start, uint32_t* sh_keys, uint32_t* sh_vals) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
-        const uint32_t dd = sort_digit(key[j], row_base, shift);
+        const uint32_t dd = sort_digit(key[j], key_base, shift);
         const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
         const uint32_t pos = (sh_start[dd] + sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
         rank2[j >> 1] = (j & 1) ? ((rank2[j >> 1] & 0xffffu) | (pos << 16))
@@ -119,7 +120,7 @@ __device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], 
 // Consecutive shared slots of one digit go to consecutive global slots
 // (destination = sh_goff[digit] + slot). Half a tile at a time: its shared
 // reads, its destinations, its stores.
-__device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, uint32_t row_base,
+__device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, uint32_t key_base,
                                            const int32_t* sh_goff, const uint32_t* sh_keys,
                                            const uint32_t* sh_vals) {
     const int tid = threadIdx.x;
@@ -136,7 +137,7 @@ __device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, ui
         }
 #pragma unroll
         for (int j = 0; j < kHalf; ++j)
-            dst[j] = sh_goff[sort_digit(key[j], row_base, S.shift)] + tid + (h * kHalf + j) * kSortThreads;
+            dst[j] = sh_goff[sort_digit(key[j], key_base, S.shift)] + tid + (h * kHalf + j) * kSortThreads;
 #pragma unroll
         for (int j = 0; j < kHalf; ++j) {
             const int i = tid + (h * kHalf + j) * kSortThreads;
@@ -173,7 +174,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     const int t = tc.table;
     const int64_t tile_base = tc.k0;
     const int tile_count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tile_base));
-    const uint32_t row_base = static_cast<uint32_t>(S.tables[t].row_base);
+    const uint32_t key_base = static_cast<uint32_t>(S.tables[t].key_base);
     const int64_t first_tile = S.table_first_tile[t];
 
     // Warp-striped load: item j of lane l is position tile_base + wid*512 + j*32 + l.
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
     }
     uint32_t rank2[kSortItems / 2];
-    rank_tile(key, tile_count, row_base, S.shift, sh_warp, rank2);
+    rank_tile(key, tile_count, key_base, S.shift, sh_warp, rank2);
     __syncthreads();
 
     // Thread d: per-warp exclusive prefix and the tile's count of digit d.
@@ -262,10 +263,10 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         static_cast<int64_t>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) + excl - start);
     __syncthreads();
 
-    scatter_tile(key, val, rank2, tile_count, row_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
+    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
     __syncthreads();
     if (sh_abort) return;
-    write_tile(S, tile_count, row_base, sh_goff, sh_keys, sh_vals);
+    write_tile(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
 }
 
 // ---------------------------------------------------------------- reduce-then-scan
@@ -280,7 +281,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_count_kernel(const SortPas
     sh[tid] = 0;
     const Chunk tc = S.tiles[tile];
     const int count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tc.k0));
-    const uint32_t rb = static_cast<uint32_t>(S.tables[tc.table].row_base);
+    const uint32_t rb = static_cast<uint32_t>(S.tables[tc.table].key_base);
     uint32_t k[kSortItems];
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
@@ -381,7 +382,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const So
     const Chunk tc = S.tiles[tile];
     const int64_t tile_base = tc.k0;
     const int tile_count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tile_base));
-    const uint32_t row_base = static_cast<uint32_t>(S.tables[tc.table].row_base);
+    const uint32_t key_base = static_cast<uint32_t>(S.tables[tc.table].key_base);
     uint32_t key[kSortItems], val[kSortItems];
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
@@ -392,7 +393,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const So
     }
     __syncthreads();
     uint32_t rank2[kSortItems / 2];
-    rank_tile(key, tile_count, row_base, S.shift, sh_warp, rank2);
+    rank_tile(key, tile_count, key_base, S.shift, sh_warp, rank2);
     __syncthreads();
     const int d = tid;
     uint32_t count = 0;
@@ -407,9 +408,9 @@ __global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const So
     sh_start[d] = static_cast<uint32_t>(start);
     sh_goff[d] = static_cast<int32_t>(static_cast<int64_t>(slot) - start);
     __syncthreads();
-    scatter_tile(key, val, rank2, tile_count, row_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
+    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
     __syncthreads();
-    write_tile(S, tile_count, row_base, sh_goff, sh_keys, sh_vals);
+    write_tile(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
 }
 
 // ---------------------------------------------------------------- single sweep
@@ -440,7 +441,7 @@ __global__ void __launch_bounds__(256) sort_hist_kernel(const uint32_t* keys, co
             __syncthreads();    // the flush is done before new counts start
             cur = tc.table;
         }
-        const uint32_t rb = static_cast<uint32_t>(tables[cur].row_base);
+        const uint32_t rb = static_cast<uint32_t>(tables[cur].key_base);
         const int len = static_cast<int>(tc.len & 0x7fffffffu);
         // All of the tile's loads first, then the counts.
         uint32_t r[kSortItems];

@@ -32,7 +32,8 @@ EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward
            "cb_tbe_get_error", "cb_tbe_last_timings", "cb_tbe_component_name",
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
            "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad",
-           "cb_tbe_backward_apply", "cb_tbe_apply_sparse", "cb_kjt_replicate")
+           "cb_tbe_backward_apply", "cb_tbe_apply_sparse", "cb_kjt_replicate",
+           "cb_tbe_sorted_payloads")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -87,11 +88,13 @@ def load_library() -> ctypes.CDLL:
     lib.cb_tbe_apply_sparse.argtypes = [p, ctypes.POINTER(CbSparseGrad), ctypes.c_int, ctypes.c_float,
                                         ctypes.c_float, p, p]
     lib.cb_kjt_replicate.argtypes = [p, p, p, ctypes.c_int, i32, i32, i64, i32, p, p, p, p]
+    lib.cb_tbe_sorted_payloads.argtypes = [p, p, i64, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
                  "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward",
-                 "cb_tbe_weight_grad", "cb_tbe_backward_apply", "cb_kjt_replicate"):
+                 "cb_tbe_weight_grad", "cb_tbe_backward_apply", "cb_kjt_replicate",
+                 "cb_tbe_sorted_payloads"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -338,6 +341,15 @@ class TBE:
                                                 _ptr(go), _ptr(out), self._stream()),
                    "cb_tbe_weight_grad")
         return out
+
+    def sorted_payloads(self, num_indices: int) -> torch.Tensor:
+        """The last backward's sorted payloads (cb_tbe_sorted_payloads) as int64 [n]:
+        lookup positions (weights or mean pooling) or bags t*B + b, in sorted order."""
+        buf = torch.empty(max(num_indices, 1), dtype=torch.int32, device=self.device)
+        with torch.cuda.device(self.device):
+            _check(self._lib.cb_tbe_sorted_payloads(self._h, _ptr(buf), num_indices, self._stream()),
+                   "cb_tbe_sorted_payloads")
+        return buf[:num_indices].to(torch.int64) & 0xffffffff
 
     def get_error(self) -> int:
         with torch.cuda.device(self.device):

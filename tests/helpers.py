@@ -187,3 +187,60 @@ def compact_tables(tables, indices, offsets, num_tables, batch):
         new_tabs.append(tables[t].index_select(0, uniq.to(tables[t].device)).cpu())
         new_ind.append(torch.searchsorted(uniq, idx).cpu())
     return new_tabs, torch.cat(new_ind).to(indices.dtype) if new_ind else indices.cpu()
+
+
+def storage_ulp(x: np.ndarray, dtype) -> np.ndarray:
+    """Spacing of the storage type at |x| (for a one-rounding allowance)."""
+    mant = {torch.float32: 23, torch.float16: 10, torch.bfloat16: 7}[dtype]
+    emin = {torch.float32: -126, torch.float16: -14, torch.bfloat16: -126}[dtype]
+    e = np.floor(np.log2(np.maximum(np.abs(x), 2.0 ** emin)))
+    return 2.0 ** (e - mant)
+
+
+def bag_of_positions(offsets) -> torch.Tensor:
+    """Bag t*B + b of every lookup position (int64 [n]), from key-major offsets."""
+    off = torch.as_tensor(offsets).cpu().to(torch.int64)
+    lens = off[1:] - off[:-1]
+    return torch.repeat_interleave(torch.arange(lens.numel(), dtype=torch.int64), lens)
+
+
+def inject_out_of_range(tables, indices, offsets, batch, seed, frac=0.05):
+    """A copy of `indices` where about `frac` of the lookups of every table hold
+    -1 or rows_t instead; returns (indices, bool mask of the replaced lookups)."""
+    g = torch.Generator().manual_seed(seed)
+    ind = indices.cpu().clone()
+    off = offsets.cpu().to(torch.int64)
+    bad = torch.rand(ind.numel(), generator=g) < frac
+    for t, E in enumerate(tables):
+        s, e = int(off[t * batch]), int(off[(t + 1) * batch])
+        sel = bad[s:e]
+        k = int(sel.sum())
+        if k == 0:
+            continue
+        hi = torch.randint(0, 2, (k,), generator=g).bool()
+        vals = torch.where(hi, torch.full((k,), int(E.shape[0])), torch.full((k,), -1))
+        part = ind[s:e]
+        part[sel] = vals.to(ind.dtype)
+    return ind, bad
+
+
+def without_lookups(indices, offsets, weights, drop, mean):
+    """The batch with the lookups where `drop` is set removed, as the library
+    treats them: they add nothing, and for mean pooling the bag length still
+    counts them. A mean-pooled batch therefore becomes a sum-pooled one whose
+    weights are w_i / L (L the original length, rounded to fp32 as the library
+    rounds its coefficient). Returns (indices, offsets, weights or None)."""
+    off = torch.as_tensor(offsets).cpu().to(torch.int64)
+    ind = torch.as_tensor(indices).cpu()
+    bag = bag_of_positions(off)
+    keep = ~drop
+    lens = off[1:] - off[:-1]
+    kept = torch.bincount(bag[keep], minlength=lens.numel())
+    new_off = torch.zeros(lens.numel() + 1, dtype=torch.int64)
+    new_off[1:] = torch.cumsum(kept, 0)
+    w = None if weights is None else torch.as_tensor(weights).cpu().to(torch.float32)
+    if mean:
+        base = torch.ones(ind.numel(), dtype=torch.float32) if w is None else w
+        w = base / lens[bag].to(torch.float32)
+    return (ind[keep].contiguous(), new_off.to(ind.dtype),
+            None if w is None else w[keep].contiguous())

@@ -88,3 +88,25 @@ def test_product_path_fails_loudly_without_the_library(monkeypatch, tmp_path):
     monkeypatch.setattr(tbe, "_lib", None)
     with pytest.raises(RuntimeError, match="missing"):
         tbe.load_library()
+
+
+def test_noalloc_refuses_sizes_that_would_wrap_the_scratch_layout(lib):
+    # num_indices near 2^63: the chunk count alone exceeds the static scratch, so the
+    # call is refused on the host before any size product can wrap around (and
+    # before any pointer is touched: these are fake, aligned addresses).
+    from paper_2609_30656_gb300 import tbe
+    f = lib.cb_tbe_forward_noalloc
+    p, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    f.argtypes = [p, i32, ctypes.c_int, ctypes.c_int, i32, p, i64, p, p, p, p]
+    f.restype = ctypes.c_int
+    descs = (tbe.CbTableDesc * 1)(tbe.CbTableDesc(4096, 10, 512, 0))
+    for n in (2**63 - 1, 2**62, 2**40):
+        assert f(descs, 1, 0, 1, 1, p(4096), n, p(8192), None, p(12288), None) == tbe.CB_ERR_CAPACITY
+
+
+def test_create_refuses_a_key_space_beyond_32_bits(lib):
+    # Every table's rows plus one spare key per table must stay below 2^32.
+    from paper_2609_30656_gb300 import tbe
+    h = ctypes.c_void_p()
+    descs = (tbe.CbTableDesc * 2)(tbe.CbTableDesc(4096, 2**31, 4, 0), tbe.CbTableDesc(4096, 2**31 - 2, 4, 0))
+    assert lib.cb_tbe_create(descs, 2, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG

@@ -194,10 +194,12 @@ def test_workload_full_size(name):
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name", ["cfg5"])
+@pytest.mark.parametrize("name", ["cfg5", "cfg5u"])
 def test_cfg5_full_size_sampled_tables(name):
     # Full 100-table batch on the GPU; three tables (first, middle, last) are
     # checked completely against the oracle run on that table's lookups alone.
+    # cfg5u (uniform indices) is the reuse-free control: ~1.7e8 distinct rows,
+    # nearly every 32-lookup batch of the reduce holds run ends.
     w = wl.get_workload(name)
     tables = wl.make_tables(w, 0, DEV)
     b = wl.make_batch(w, 0, DEV)

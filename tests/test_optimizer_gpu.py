@@ -8,7 +8,7 @@ import torch
 
 import oracle
 from tests.conftest import parse_value
-from tests.helpers import backward_reference, random_problem, table_meta
+from tests.helpers import backward_reference, random_problem, storage_ulp, table_meta
 from paper_2609_30656_gb300 import workloads as wl
 
 pytestmark = pytest.mark.gpu
@@ -16,12 +16,7 @@ DEV = torch.device("cuda:0")
 U32 = 2.0 ** -24
 
 
-def _ulp(x: np.ndarray, dtype) -> np.ndarray:
-    """Spacing of the storage type at |x| (for a one-rounding allowance)."""
-    mant = {torch.float32: 23, torch.float16: 10, torch.bfloat16: 7}[dtype]
-    emin = {torch.float32: -126, torch.float16: -14, torch.bfloat16: -126}[dtype]
-    e = np.floor(np.log2(np.maximum(np.abs(x), 2.0 ** emin)))
-    return 2.0 ** (e - mant)
+_ulp = storage_ulp
 
 
 def _run(tables, batch, ind, off, go, w, mean, optimizer, lr, eps=1e-8, state=None, two_pass=False):
