@@ -248,9 +248,21 @@ def cpu_threads() -> int:
 
 # ----------------------------------------------------------------------------- GPU arm
 
-def run_ours(args):
-    import numpy as np
+def quantile(xs, q: float) -> float:
+    """Linear-interpolated quantile of a non-empty sample."""
+    s = sorted(xs)
+    k = (len(s) - 1) * q
+    lo, hi = math.floor(k), math.ceil(k)
+    return s[lo] + (s[hi] - s[lo]) * (k - lo)
 
+
+def timing_summary(ms):
+    return {"median": round(statistics.median(ms), 4), "p10": round(quantile(ms, 0.1), 4),
+            "p90": round(quantile(ms, 0.9), 4), "mean": round(statistics.mean(ms), 4),
+            "samples": len(ms)}
+
+
+def run_ours(args):
     from paper_2609_30656_gb300 import tbe
 
     world, rank, local = dist_env()
@@ -264,7 +276,9 @@ def run_ours(args):
     batches = [wl.make_batch(w, seed + 1000 * rank, dev, batch_index=k) for k in range(args.rotate)]
     grads_out = [wl.make_grad_out(w, seed + 1000 * rank, dev, batch_index=k)
                  for k in range(args.rotate)]
-    m = tbe.TBE(tables, pooling="mean" if w.mean else "sum", timing=True)
+    # The headline handle records no per-component events: the timed steps carry
+    # nothing but the kernels. The breakdown below uses a second handle.
+    m = tbe.TBE(tables, pooling="mean" if w.mean else "sum")
     max_n = max(b.num_indices for b in batches)
     m.reserve(w.batch, max_n)
     out = torch.empty(w.batch, w.sum_dims, dtype=torch.float32, device=dev)
@@ -295,10 +309,8 @@ def run_ours(args):
         raise RuntimeError("device-side error during warm-up")
     torch.cuda.synchronize()
 
-    names = tbe.component_names()
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    comp = {n: [] for n in names}
     launches0 = m.launch_count()
     if world > 1:
         torch.distributed.barrier()
@@ -310,8 +322,6 @@ def run_ours(args):
             starts[k].record()
             step(args.warmup + k)
             stops[k].record()
-            for n_, v in m.last_timings().items():
-                comp[n_].append(v)
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
     if world > 1:
@@ -320,11 +330,10 @@ def run_ours(args):
     if m.get_error() != 0:
         raise RuntimeError("device-side error during the timed steps")
     step_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
-    ms = sum(step_ms) / len(step_ms)
+    ms = statistics.median(step_ms)
 
     # Work of the timed steps (host-side sizes).
     fwd_b, bwd_b, rows_g = 0.0, 0.0, 0.0
-    comp_bytes = {n: 0.0 for n in names}
     uniq_fwd = 0.0
     for k in range(args.steps):
         i = (args.warmup + k) % args.rotate
@@ -333,55 +342,46 @@ def run_ours(args):
         bwd_b += metrics.backward_bytes(c, uniq_tables[i])["total"]
         uniq_fwd += metrics.forward_unique_bytes(c, uniq_tables[i])
         rows_g += 2 * c.n
-        for n_, v in metrics.component_bytes(c, uniq_tables[i], w.rows, packed).items():
-            comp_bytes[n_] += v
     per_step_bytes = (fwd_b + bwd_b) / args.steps
     tot_ms, tot_bytes, tot_rows = aggregate(ms, per_step_bytes, rows_g / args.steps, world)
     gbs = tot_bytes / (tot_ms * 1e-3) / 1e9
     peak, peak_kind = measured_hbm_peak()
 
-    comp_ms = {n: statistics.mean(v) for n, v in comp.items() if v and min(v) >= 0}
-    fwd_ms = comp_ms["fwd.prep"] + comp_ms["fwd.gather"] + comp_ms["fwd.fixup"]
-    bwd_ms = sum(comp_ms[n] for n in names if n.startswith("bwd."))
+    # Per-component breakdown: a separate run with CB_TIMING events between the
+    # components, so the headline above carries no event overhead.
+    comp_ms, comp_bytes, comp_compulsory = run_breakdown(args, w, tables, batches, grads_out, g, out,
+                                                         flush, counts, uniq_tables, packed)
+    names = tbe.component_names()
+    fwd_ms = sum(comp_ms[n] for n in names if n.startswith("fwd.") and n in comp_ms)
+    bwd_ms = sum(comp_ms[n] for n in names if n.startswith("bwd.") and n in comp_ms)
     components = {}
     for n in names:
         if n not in comp_ms:
             continue
-        cb = comp_bytes.get(n)
         entry = {"ms": round(comp_ms[n], 4), "share": round(comp_ms[n] / (fwd_ms + bwd_ms), 4)}
-        if cb:
-            entry["alg_gbs"] = round(cb / args.steps / (comp_ms[n] * 1e-3) / 1e9, 1)
+        if comp_bytes.get(n):
+            entry["alg_gbs"] = round(comp_bytes[n] / (comp_ms[n] * 1e-3) / 1e9, 1)
         components[n] = entry
-    dominant = max((n for n in comp_bytes if n in comp_ms), key=lambda n: comp_ms[n])
-    dom_bytes = comp_bytes[dominant] / args.steps
-    achieved = dom_bytes / (comp_ms[dominant] * 1e-3) / 1e9
-    traffic = recorded_traffic(dominant, w.name)
-    roofline = {"bound": "hbm", "kernel": dominant, "achieved": round(achieved, 1),
-                "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
-                else "fallback 6800 GB/s",
-                "traffic": traffic,
-                "bytes_per_launch": int(dom_bytes)}
-    if traffic:
-        dram = traffic / (comp_ms[dominant] * 1e-3) / 1e9
-        roofline["achieved_dram"] = round(dram, 1)
-        roofline["frac_dram"] = round(dram / peak, 4)
-        roofline["note"] = ("achieved counts every lookup's row (algorithmic bytes); repeated rows "
-                            "are served from L2/L1, so it can exceed the HBM copy bandwidth; "
-                            "traffic is the measured DRAM bytes per launch")
+    ceiling = None if args.no_l2 else run_l2_ceiling(dev)
+    roofline = roofline_of(w.name, comp_ms, comp_bytes, comp_compulsory, peak, peak_kind, ceiling,
+                           counts, w)
     mean_counts_n = statistics.mean(c.n for c in counts)
     fwd_bytes_step = fwd_b / args.steps
     bwd_bytes_step = bwd_b / args.steps
     line = {
         "metric": METRIC, "value": round(gbs, 1), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(tot_ms, 4),
+        "step_ms": timing_summary(step_ms),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f32", "storage_dtype": w.dtype, "data": "synthetic",
         "config": {"workload": describe(w),
                    "l2": f"flushed before every step ({2 * l2 >> 20} MB write, outside the "
                          "step's events); inputs also exceed L2",
                    "rotating_batches": args.rotate, "seed": seed,
-                   "lookups_per_step": int(mean_counts_n), "parallelism": f"replicas x{world}"},
+                   "lookups_per_step": int(mean_counts_n), "parallelism": f"replicas x{world}",
+                   "timing": "value and ms_per_step: the median of the per-step CUDA-event times "
+                             "(p10/p90 in step_ms) on a handle without component events; "
+                             "components: a separate run with CB_TIMING events"},
         "pct_hbm": round(gbs / world / peak, 4), "pct_hbm_nominal": round(gbs / world / NOMINAL_HBM_GBS, 4),
         "rows_per_s": round(tot_rows / (tot_ms * 1e-3), 1),
         "fwd": {"ms": round(fwd_ms, 4), "alg_gbs": round(fwd_bytes_step / (fwd_ms * 1e-3) / 1e9, 1),
@@ -397,10 +397,9 @@ def run_ours(args):
         "wall_ms_per_step": round(wall * 1e3 / args.steps, 3),
         "clocks": clk.summary(),
     }
+    if ceiling:
+        line["l2_ceiling"] = ceiling
 
-    # The reuse-free control: the forward over uniform indices on the same tables.
-    if w.zipf_alpha is not None and not args.no_control:
-        line["control_uniform"] = run_control(args, m, w, dev, out, flush, world, peak)
     # Next rows: the FM cross term and its gradient on the same pooled output,
     # and the gradient of the per-sample weights on the first batch.
     if not args.no_next:
@@ -424,47 +423,194 @@ def run_ours(args):
     # The oracle on the host cores, rank 0 only, single GPU runs only.
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(args, w, tables, batches[0], grads_out[0])
+    # The reuse-free control: the whole step over uniform indices on the same
+    # tables (last: it needs room for ~1.7e8 gradient rows).
+    if w.zipf_alpha is not None and not args.no_control:
+        go0 = grads_out[0]
+        b = go = probe = None
+        del g, out, batches, grads_out, b, go, probe
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        line["control_uniform"] = run_control(args, m, w, dev, flush, peak, go0, tables)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
 
 
-def run_control(args, m, w, dev, out, flush, world, peak):
-    """Forward gather-pool on uniform indices over the same tables (no row reuse)."""
+def run_breakdown(args, w, tables, batches, grads_out, g, out, flush, counts, uniq_tables, packed,
+                  steps=None):
+    """Median per-component times (CB_TIMING events between the components) over a
+    few steps on a second handle, with their algorithmic and compulsory bytes."""
+    from paper_2609_30656_gb300 import tbe
+    mt = tbe.TBE(tables, pooling="mean" if w.mean else "sum", timing=True)
+    steps = steps or args.breakdown_steps
+    rot = len(batches)
+    comp = {}
+    comp_bytes, comp_compulsory = {}, {}
+    for k in range(2 + steps):
+        i = k % rot
+        b, go = batches[i], grads_out[i]
+        flush.zero_()
+        mt.forward(b.indices, b.offsets, b.weights, out=out)
+        fwd_t = mt.last_timings()
+        mt.backward_into(g, b.indices, b.offsets, go, b.weights)
+        t = mt.last_timings()
+        if k < 2:
+            continue
+        for n_, v in t.items():
+            v = fwd_t[n_] if n_.startswith("fwd.") else v
+            if v >= 0:
+                comp.setdefault(n_, []).append(v)
+        cb = metrics.component_bytes(counts[i], uniq_tables[i], w.rows, packed)
+        cc = metrics.component_compulsory_bytes(counts[i], uniq_tables[i], packed)
+        for n_, v in cb.items():
+            comp_bytes[n_] = comp_bytes.get(n_, 0.0) + v / steps
+        for n_, v in cc.items():
+            comp_compulsory[n_] = comp_compulsory.get(n_, 0.0) + v / steps
+    if mt.get_error() != 0:
+        raise RuntimeError("device-side error in the component breakdown")
+    mt.close()
+    return ({n_: statistics.median(v) for n_, v in comp.items()}, comp_bytes, comp_compulsory)
+
+
+def roofline_of(workload, comp_ms, comp_bytes, comp_compulsory, peak, peak_kind, ceiling, counts, w):
+    """The roofline object of the dominant kernel: the fraction of the HBM copy
+    bandwidth its DRAM traffic reaches (ncu bytes per launch, when recorded for
+    the current sources, else its compulsory bytes), with the algorithmic and
+    L2-gather figures beside it under their own names."""
+    dominant = max((n for n in comp_bytes if n in comp_ms), key=lambda n: comp_ms[n])
+    t = comp_ms[dominant] * 1e-3
+    alg = comp_bytes[dominant]
+    comp = comp_compulsory.get(dominant)
+    traffic = recorded_traffic(dominant, workload)
+    if traffic:
+        achieved, basis = traffic / t / 1e9, "dram"
+    else:
+        achieved, basis = comp / t / 1e9, "compulsory"
+    r = {"bound": "hbm", "kernel": dominant, "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+         "frac": round(achieved / peak, 4), "basis": basis,
+         "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+         else "fallback 6800 GB/s",
+         "traffic": traffic, "launch_ms": round(comp_ms[dominant], 4),
+         "compulsory_bytes_per_launch": int(comp) if comp else None,
+         "compulsory_frac": round(comp / t / 1e9 / peak, 4) if comp else None,
+         "alg_bytes_per_launch": int(alg), "alg_gbs": round(alg / t / 1e9, 1),
+         "alg_frac": round(alg / t / 1e9 / peak, 4),
+         "note": "achieved/frac: DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum, "
+                 "when recorded for the current sources; else the compulsory bytes: every distinct "
+                 "row or grad_out slice once) over the launch's event time; alg_*: every lookup's "
+                 "row counted, which exceeds HBM bandwidth when L2 serves the repeats"}
+    if ceiling:
+        # The gathered part of the kernel against the L2 random-gather rate
+        # of rows of the same size.
+        if dominant == "bwd.reduce":
+            gathered = sum(metrics.backward_bytes(c, [0] * c.num_tables)["grad_gather"] for c in counts) / len(counts)
+            row = 4 * max(w.dims)
+        else:
+            gathered = sum(metrics.forward_bytes(c)["rows"] for c in counts) / len(counts)
+            row = w.elem_bytes * max(w.dims)
+        key = str(min(512, row))
+        if key in ceiling:
+            r["l2_gather_gbs"] = round(gathered / t / 1e9, 1)
+            r["frac_l2"] = round(gathered / t / 1e9 / ceiling[key]["gbs"], 4)
+            r["l2_ceiling_row_bytes"] = int(key)
+    return r
+
+
+def run_l2_ceiling(dev, reps: int = 5):
+    """cb_gather_ceiling on a 33.5 MB row set (one cfg5 table's grad_out slice,
+    [65536, 128] fp32) for 512- and 256-byte rows: 2^25 uniformly random rows
+    per launch, the median of `reps` launches after two warm-ups."""
+    from paper_2609_30656_gb300 import tbe
+    g = torch.Generator(device=dev)
+    g.manual_seed(5)
+    n = 1 << 25
+    res = {}
+    for row_bytes in (512, 256):
+        R = (65536 * 512) // row_bytes
+        rows = torch.randn(R, row_bytes // 4, generator=g, device=dev)
+        idx = torch.randint(0, R, (n,), generator=g, device=dev, dtype=torch.int32)
+        out = torch.empty((n + 31) // 32, dtype=torch.float32, device=dev)
+        for _ in range(2):
+            tbe.gather_ceiling(rows, idx, out)
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        for a, b in ev:
+            a.record()
+            tbe.gather_ceiling(rows, idx, out)
+            b.record()
+        torch.cuda.synchronize()
+        ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+        res[str(row_bytes)] = {"gbs": round(n * row_bytes / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
+                               "rows": n, "set_mb": round(R * row_bytes / 1e6, 1)}
+        del rows, idx, out
+    res["how"] = ("cb_gather_ceiling: one warp per 32 random rows of an L2-resident set, 16 bytes per "
+                  "lane, 8 row steps in flight (the walkers' load shape without their bookkeeping)")
+    return res
+
+
+def run_control(args, m, w, dev, flush, peak, go, tables):
+    """The whole step (forward + de-duplicated backward) on uniform indices over
+    the same tables: no row reuse, so algorithmic bytes ~ DRAM traffic."""
+    from paper_2609_30656_gb300 import tbe
     wu = dataclasses.replace(w, zipf_alpha=None)
     batches = [wl.make_batch(wu, args.seed + 7, dev, batch_index=k) for k in range(2)]
     counts = [metrics.batch_counts(w.dims, w.elem_bytes, w.batch, b.offsets, b.weights is not None)
               for b in batches]
+    U_max, F_max, uniq = 0, 0, []
+    for b in batches:
+        probe = m.alloc_grad(0, 0, size_only=True)
+        m.backward_into(probe, b.indices, b.offsets, go, b.weights)
+        U_max, F_max = max(U_max, probe.num_unique), max(F_max, probe.num_floats)
+        toff = probe.table_offsets.cpu().tolist()
+        uniq.append([toff[t + 1] - toff[t] for t in range(w.num_tables)])
+    g = m.alloc_grad(U_max, F_max)
+    out = torch.empty(w.batch, w.sum_dims, dtype=torch.float32, device=dev)
     for k in range(3):
         b = batches[k % 2]
         m.forward(b.indices, b.offsets, b.weights, out=out)
+        m.backward_into(g, b.indices, b.offsets, go, b.weights)
     torch.cuda.synchronize()
     steps = 6
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(steps)]
-    gather_ms = []
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
     for k in range(steps):
         b = batches[k % 2]
         flush.zero_()
         ev[k][0].record()
         m.forward(b.indices, b.offsets, b.weights, out=out)
         ev[k][1].record()
-        gather_ms.append(m.last_timings()["fwd.gather"])
+        m.backward_into(g, b.indices, b.offsets, go, b.weights)
+        ev[k][2].record()
     torch.cuda.synchronize()
-    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
-    nbytes = statistics.mean(metrics.forward_bytes(counts[k % 2])["total"] for k in range(steps))
-    gms = statistics.mean(gather_ms)
-    res = {"workload": describe(wu).replace("cfg5:", "cfg5u (same tables):", 1),
-           "fwd_ms": round(ms, 4), "fwd_alg_gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
-           "fwd_pct_hbm": round(nbytes / (ms * 1e-3) / 1e9 / peak, 4),
-           "gather_ms": round(gms, 4),
-           "gather_alg_gbs": round(nbytes / (gms * 1e-3) / 1e9, 1)}
-    traffic = recorded_traffic("fwd.gather", "cfg5u")
-    res["gather_traffic"] = traffic
-    if traffic:
-        res["gather_frac_dram"] = round(traffic / (gms * 1e-3) / 1e9 / peak, 4)
-    del batches
+    if m.get_error() != 0:
+        raise RuntimeError("device-side error in the uniform-index control")
+    fwd = statistics.median(e[0].elapsed_time(e[1]) for e in ev)
+    bwd = statistics.median(e[1].elapsed_time(e[2]) for e in ev)
+    stp = statistics.median(e[0].elapsed_time(e[2]) for e in ev)
+    fb = statistics.mean(metrics.forward_bytes(counts[k % 2])["total"] for k in range(steps))
+    bb = statistics.mean(metrics.backward_bytes(counts[k % 2], uniq[k % 2])["total"] for k in range(steps))
+    comp_ms, comp_bytes, comp_compulsory = run_breakdown(
+        args, w, tables, batches, [go, go], g, out, flush, counts, uniq, w.weighted or w.mean, steps=4)
+    res = {"workload": describe(wu).replace(f"{w.name}:", "cfg5u (same tables):", 1),
+           "step_ms": round(stp, 4), "step_alg_gbs": round((fb + bb) / (stp * 1e-3) / 1e9, 1),
+           "step_pct_hbm": round((fb + bb) / (stp * 1e-3) / 1e9 / peak, 4),
+           "fwd_ms": round(fwd, 4), "fwd_alg_gbs": round(fb / (fwd * 1e-3) / 1e9, 1),
+           "fwd_pct_hbm": round(fb / (fwd * 1e-3) / 1e9 / peak, 4),
+           "bwd_ms": round(bwd, 4), "bwd_alg_gbs": round(bb / (bwd * 1e-3) / 1e9, 1),
+           "bwd_pct_hbm": round(bb / (bwd * 1e-3) / 1e9 / peak, 4),
+           "unique_rows": int(sum(uniq[0])),
+           "components": {n: round(v, 4) for n, v in comp_ms.items()}}
+    for kern in ("fwd.gather", "bwd.reduce"):
+        t = comp_ms[kern] * 1e-3
+        e = {"ms": round(comp_ms[kern], 4), "alg_gbs": round(comp_bytes[kern] / t / 1e9, 1),
+             "alg_frac": round(comp_bytes[kern] / t / 1e9 / peak, 4)}
+        traffic = recorded_traffic(kern, "cfg5u")
+        e["traffic"] = traffic
+        if traffic:
+            e["frac_dram"] = round(traffic / t / 1e9 / peak, 4)
+        res[kern] = e
+    del batches, g, out
     return res
 
 
@@ -631,7 +777,7 @@ def write_report(path, w, line, comp_ms, comp_bytes, counts, uniq_tables, peak):
     for c, u in zip(counts, uniq_tables):
         for k, v in metrics.component_flops(c, u, w.mean).items():
             flops[k] = flops.get(k, 0.0) + v / steps
-    per_bytes = {k: v / line["steps"] for k, v in comp_bytes.items()}
+    per_bytes = dict(comp_bytes)  # per step already (the breakdown run's mean)
     extra = {}
     nxt = line.get("next_rows", {})
     if "fm" in nxt:
@@ -692,54 +838,81 @@ def run_fm_only(args):
 
 
 def run_e2e(args, m, w, batches, grads_out, g, out, dev, world):
-    """Forward + backward of a host batch, every step copying its inputs from pinned
-    host memory and reading its result back. Timed twice: serially (the binding copies
-    the host tensors it is given, on the compute stream) and pipelined (each step's
-    inputs copied once, on a copy stream, into one of two device buffers while the
-    previous step computes); the pipelined figure is the line's e2e value."""
+    """Forward + backward of a host batch through the public API, every step
+    copying its inputs from pinned host memory and its results back to pinned
+    host memory: the pooled output [B, sum D] and the row-sparse gradient (ids,
+    offsets, values). The value is the pipelined figure: inputs copied on one
+    stream into double-buffered device inputs while the previous step computes,
+    results copied back on another stream from double-buffered device outputs
+    while the next step computes. Also reported: the same with the results left
+    on the device (only their sizes read back), and the binding's own serial
+    path (host tensors copied on the compute stream, results read after it)."""
     b, go = batches[0], grads_out[0]
     h_ind = b.indices.cpu().pin_memory()
     h_off = b.offsets.cpu().pin_memory()
     h_w = None if b.weights is None else b.weights.cpu().pin_memory()
     h_go = go.cpu().pin_memory()
-    h_res = torch.empty(2 + w.num_tables + 1, dtype=torch.int64).pin_memory()
     steps = max(2, args.steps if args.e2e_steps is None else min(args.steps, args.e2e_steps))
     bytes_in = (h_ind.numel() * 8 + h_off.numel() * 8 + (0 if h_w is None else h_w.numel() * 4)
                 + h_go.numel() * 4)
-    bytes_out = h_res.numel() * 8
+    # This batch's result sizes (from an untimed call): a caller reads the two
+    # device scalars to size its copies; here they are fixed for the batch.
+    m.forward(b.indices, b.offsets, b.weights, out=out)
+    m.backward_into(g, b.indices, b.offsets, go, b.weights)
+    U, F = g.num_unique, g.num_floats
+    T = w.num_tables
+    h_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    h_ids = torch.empty(U, dtype=torch.int64).pin_memory()
+    h_goff = torch.empty(U + 1, dtype=torch.int64).pin_memory()
+    h_grads = torch.empty(F, dtype=torch.float32).pin_memory()
+    h_small = torch.empty(2 + T + 1, dtype=torch.int64).pin_memory()
+    bytes_out_full = (h_out.numel() * 4 + h_ids.numel() * 8 + h_goff.numel() * 8 + h_grads.numel() * 4
+                      + h_small.numel() * 8)
+    bytes_out_sizes = h_small.numel() * 8
 
-    def read_result():
-        h_res[0:1].copy_(g.num_unique_dev, non_blocking=True)
-        h_res[1:2].copy_(g.num_floats_dev, non_blocking=True)
-        h_res[2:].copy_(g.table_offsets, non_blocking=True)
+    def read_sizes(gg):
+        h_small[0:1].copy_(gg.num_unique_dev, non_blocking=True)
+        h_small[1:2].copy_(gg.num_floats_dev, non_blocking=True)
+        h_small[2:].copy_(gg.table_offsets, non_blocking=True)
+
+    def read_all(gg, yy):
+        read_sizes(gg)
+        h_out.copy_(yy, non_blocking=True)
+        h_ids.copy_(gg.unique_ids[:U], non_blocking=True)
+        h_goff.copy_(gg.grad_offsets[:U + 1], non_blocking=True)
+        h_grads.copy_(gg.grads[:F], non_blocking=True)
 
     def serial_step():
         # The user's call with host tensors: the binding copies them to the device.
         m.forward(h_ind, h_off, h_w, out=out)
         m.backward_into(g, h_ind, h_off, h_go, h_w)
-        read_result()
+        read_all(g, out)
 
     compute = torch.cuda.current_stream(dev)
-    copy = torch.cuda.Stream(dev)
-    bufs = [{"ind": torch.empty_like(h_ind, device=dev), "off": torch.empty_like(h_off, device=dev),
-             "w": None if h_w is None else torch.empty_like(h_w, device=dev),
-             "go": torch.empty_like(h_go, device=dev)} for _ in range(2)]
+    copy_in = torch.cuda.Stream(dev)
+    copy_out = torch.cuda.Stream(dev)
+    ins = [{"ind": torch.empty_like(h_ind, device=dev), "off": torch.empty_like(h_off, device=dev),
+            "w": None if h_w is None else torch.empty_like(h_w, device=dev),
+            "go": torch.empty_like(h_go, device=dev)} for _ in range(2)]
+    outs = [(g, out), (m.alloc_grad(g.unique_ids.numel(), g.grads.numel()), torch.empty_like(out))]
     copied = [torch.cuda.Event() for _ in range(2)]
-    done = [torch.cuda.Event() for _ in range(2)]
+    consumed = [torch.cuda.Event() for _ in range(2)]  # the step that read this input slot is done
+    computed = [torch.cuda.Event() for _ in range(2)]
+    drained = [torch.cuda.Event() for _ in range(2)]   # this output slot's results are on the host
 
     def stage(slot):
-        copy.wait_event(done[slot])  # the step that last read this buffer has finished
-        with torch.cuda.stream(copy):
-            d = bufs[slot]
+        copy_in.wait_event(consumed[slot])
+        with torch.cuda.stream(copy_in):
+            d = ins[slot]
             d["ind"].copy_(h_ind, non_blocking=True)
             d["off"].copy_(h_off, non_blocking=True)
             if h_w is not None:
                 d["w"].copy_(h_w, non_blocking=True)
             d["go"].copy_(h_go, non_blocking=True)
-            copied[slot].record(copy)
+            copied[slot].record(copy_in)
 
-    def pipelined(n):
-        for e in done:
+    def pipelined(n, full):
+        for e in consumed + drained:
             e.record(compute)
         stage(0)
         for k in range(n):
@@ -747,18 +920,27 @@ def run_e2e(args, m, w, batches, grads_out, g, out, dev, world):
             if k + 1 < n:
                 stage((k + 1) % 2)  # the next step's inputs, while this step computes
             compute.wait_event(copied[slot])
-            d = bufs[slot]
-            m.forward(d["ind"], d["off"], d["w"], out=out)
-            m.backward_into(g, d["ind"], d["off"], d["go"], d["w"])
-            read_result()
-            done[slot].record(compute)
+            compute.wait_event(drained[slot])  # step k - 2's results have left this slot
+            d = ins[slot]
+            gg, yy = outs[slot]
+            m.forward(d["ind"], d["off"], d["w"], out=yy)
+            m.backward_into(gg, d["ind"], d["off"], d["go"], d["w"])
+            consumed[slot].record(compute)
+            computed[slot].record(compute)
+            copy_out.wait_event(computed[slot])
+            with torch.cuda.stream(copy_out):
+                if full:
+                    read_all(gg, yy)
+                else:
+                    read_sizes(gg)
+                drained[slot].record(copy_out)
 
     serial_step()
-    pipelined(2)
+    pipelined(2, True)
     torch.cuda.synchronize()
     counts = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, b.offsets, b.weights is not None)
     toff = g.table_offsets.cpu().tolist()
-    uniq = [toff[t + 1] - toff[t] for t in range(w.num_tables)]
+    uniq = [toff[t + 1] - toff[t] for t in range(T)]
     step_bytes = metrics.forward_bytes(counts)["total"] + metrics.backward_bytes(counts, uniq)["total"]
 
     def timed(fn):
@@ -771,19 +953,27 @@ def run_e2e(args, m, w, batches, grads_out, g, out, dev, world):
         return (time.perf_counter() - t0) / steps
 
     el_serial = timed(lambda: [serial_step() for _ in range(steps)])
-    el_pipe = timed(lambda: pipelined(steps))
-    tot_ms, tot_bytes, _ = aggregate(el_pipe * 1e3, step_bytes, 0.0, world)
+    el_full = timed(lambda: pipelined(steps, True))
+    el_dev = timed(lambda: pipelined(steps, False))
+    tot_ms, tot_bytes, _ = aggregate(el_full * 1e3, step_bytes, 0.0, world)
+    dev_ms, _, _ = aggregate(el_dev * 1e3, step_bytes, 0.0, world)
     ser_ms, _, _ = aggregate(el_serial * 1e3, step_bytes, 0.0, world)
-    del bufs
+    if m.get_error() != 0:
+        raise RuntimeError("device-side error in the end-to-end run")
+    del ins, outs
     return {"value": round(tot_bytes / (tot_ms * 1e-3) / 1e9, 1), "unit": "GB/s",
             "ms_per_step": round(tot_ms, 3), "steps": steps,
-            "h2d_bytes_per_step": int(bytes_in), "d2h_bytes_per_step": int(bytes_out),
+            "h2d_bytes_per_step": int(bytes_in), "d2h_bytes_per_step": int(bytes_out_full),
             "serial_ms_per_step": round(ser_ms, 3),
-            "note": "every step copies its host batch (indices, offsets, weights) and grad_out "
-                    "from pinned memory and reads num_unique, num_floats and table_offsets back; "
-                    "value: copies on a second stream into double-buffered device inputs, "
-                    "overlapping the previous step's compute; serial_ms_per_step: the binding "
-                    "copying the host tensors on the compute stream"}
+            "result_on_device": {"value": round(tot_bytes / (dev_ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+                                 "ms_per_step": round(dev_ms, 3), "d2h_bytes_per_step": int(bytes_out_sizes)},
+            "note": "every step copies its host batch (indices, offsets, weights) and grad_out from "
+                    "pinned memory and copies the pooled output and the row-sparse gradient (ids, "
+                    "offsets, values, sizes) back to pinned memory; value: inputs and results on two "
+                    "copy streams with double-buffered device buffers, overlapping the neighbouring "
+                    "steps' compute; result_on_device: the same with only the sizes read back; "
+                    "serial_ms_per_step: the binding copying host tensors on the compute stream, "
+                    "results read after it"}
 
 
 def run_cpu_baseline(args, w, tables, batch0, go0, budget_s: float | None = None):
@@ -792,11 +982,44 @@ def run_cpu_baseline(args, w, tables, batch0, go0, budget_s: float | None = None
     host_tabs, ind, off, wt, go, counts = sample_problem(w, tables, batch0, go0, ntab)
     el, res = oracle_step(host_tabs, ind, off, wt, go, w.batch, w.mean, threads)
     nbytes = sample_bytes(counts, res, w.rows[:ntab])
-    return {"value": round(nbytes / el / 1e9, 3), "unit": "GB/s", "cores": threads,
-            "kind": "oracle",
-            "sample": f"forward + backward of tables 0..{ntab - 1} of {w.num_tables} at the full "
-                      f"batch ({counts.n:,} lookups, {nbytes / 1e9:.2f} GB algorithmic), "
-                      f"{el:.1f} s on {threads} threads (OpenMP over bags; the sort is serial)"}
+    out = {"value": round(nbytes / el / 1e9, 3), "unit": "GB/s", "cores": threads,
+           "kind": "oracle",
+           "sample": f"forward + backward of tables 0..{ntab - 1} of {w.num_tables} at the full "
+                     f"batch ({counts.n:,} lookups, {nbytes / 1e9:.2f} GB algorithmic), "
+                     f"{el:.1f} s on {threads} threads (OpenMP over bags; the sort is serial)"}
+    if not args.no_one_core:
+        out["one_core"] = run_one_core(args, tables[0].device)
+    return out
+
+
+def run_one_core(args, dev):
+    """The oracle on one host core over the whole of configs 1-3 (forward only for
+    config 1, as it is specified), and on all cores beside it."""
+    res = {}
+    for name in ("cfg1", "cfg2", "cfg3"):
+        w = wl.get_workload(name)
+        tables = wl.make_tables(w, args.seed, dev)
+        b = wl.make_batch(w, args.seed, dev)
+        go = wl.make_grad_out(w, args.seed, dev)
+        host_tabs, ind, off, wt, go_h, counts = sample_problem(w, tables, b, go, w.num_tables)
+        del tables, b, go
+        entry = {"lookups": counts.n}
+        for cores in (1, cpu_threads()):
+            if name == "cfg1":
+                import oracle
+                t0 = time.perf_counter()
+                oracle.forward(host_tabs, w.batch, ind, off, weights=wt, mean=w.mean, threads=cores)
+                el = time.perf_counter() - t0
+                nb = metrics.forward_bytes(counts)["total"]
+            else:
+                el, r = oracle_step(host_tabs, ind, off, wt, go_h, w.batch, w.mean, cores)
+                nb = sample_bytes(counts, r, w.rows)
+            key = "one_core" if cores == 1 else f"{cores}_cores"
+            entry[key] = {"ms": round(el * 1e3, 3), "gbs": round(nb / el / 1e9, 4),
+                          "rows_per_s": round(counts.n * (1 if name == "cfg1" else 2) / el, 1)}
+        entry["what"] = "forward" if name == "cfg1" else "forward + backward"
+        res[name] = entry
+    return res
 
 
 # ----------------------------------------------------------------------------- reference arm
@@ -872,7 +1095,12 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-control", action="store_true",
-                    help="skip the forward on uniform indices over the same tables")
+                    help="skip the step on uniform indices over the same tables")
+    ap.add_argument("--no-l2", action="store_true", help="skip the L2 random-gather ceiling leg")
+    ap.add_argument("--no-one-core", action="store_true",
+                    help="skip the one-core oracle timing of configs 1-3")
+    ap.add_argument("--breakdown-steps", type=int, default=5,
+                    help="steps of the per-component breakdown run (CB_TIMING handle)")
     ap.add_argument("--no-next", action="store_true",
                     help="skip the next-row measurements (FM cross term)")
     ap.add_argument("--report", default=None,

@@ -209,6 +209,24 @@ uint64_t cb_tbe_launch_count(const cb_tbe* h);
  * CB_ERR_INVALID_ARG when no such payloads are held. */
 cb_status cb_tbe_sorted_payloads(const cb_tbe* h, uint32_t* out, int64_t num_indices, cudaStream_t stream);
 
+/* Measurement aid (not in the paper): the rate at which this GPU gathers
+ * random rows out of a row set that fits in L2 (on skewed indices most rows
+ * the forward gather and the backward reduce read come from L2, so this rate
+ * bounds them besides the HBM bandwidth). One warp per 32 items, each lane
+ * loading one 4-byte index and 16 bytes of a row per step, 8 steps in flight,
+ * as those kernels load; it sums what it loads and writes one sum per 32 items.
+ *   rows         device [num_rows rows of row_bytes], 16-byte aligned, read as fp32
+ *   num_rows     1 .. 2^32
+ *   row_bytes    64, 128, 256 or 512
+ *   indices      device uint32 [num_indices] row numbers (a number >= num_rows
+ *                reads row 0)
+ *   out          device fp32 [ceil(num_indices / 32)]: out[k] = the sum of every
+ *                value of the rows of items 32k .. 32k + 31 (fp32, any order)
+ * CB_ERR_INVALID_ARG for a bad size or pointer; CB_ERR_CUDA if the launch fails.
+ * The rate is num_indices * row_bytes over the time of the call on `stream`. */
+cb_status cb_gather_ceiling(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* indices,
+                            int64_t num_indices, float* out, cudaStream_t stream);
+
 /* Short English description of a status code. */
 const char* cb_tbe_status_string(cb_status s);
 

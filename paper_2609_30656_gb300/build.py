@@ -22,7 +22,7 @@ LIB = os.path.join(HERE, "libcb_tbe.so")
 SOURCES = ["cb_tbe.cu", "tbe_plan.cu", "tbe_forward.cu", "tbe_forward_f32.cu", "tbe_forward_f16.cu",
            "tbe_forward_bf16.cu", "tbe_backward.cu", "tbe_sort.cu", "cb_tbe_noalloc.cu",
            "fm_interaction.cu", "tbe_weight_grad.cu", "tbe_backward_apply.cu", "kjt_replicate.cu",
-           "tbe_reduce_f16.cu", "tbe_reduce_bf16.cu", "tbe_reduce_f32.cu"]
+           "tbe_reduce_f16.cu", "tbe_reduce_bf16.cu", "tbe_reduce_f32.cu", "gather_ceiling.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

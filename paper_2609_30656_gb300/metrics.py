@@ -36,6 +36,7 @@ class BatchCounts:
     idx_bytes: int
     weighted: bool
     lookups_per_table: tuple[int, ...]
+    nonempty_per_table: tuple[int, ...] = ()  # bags with at least one lookup
 
     @property
     def n(self) -> int:
@@ -51,7 +52,13 @@ def batch_counts(dims, elem_bytes: int, batch: int, offsets: torch.Tensor, weigh
     T = len(dims)
     starts = offsets[::batch][:T + 1].to("cpu").tolist() if batch > 0 else [0] * (T + 1)
     per = tuple(int(starts[t + 1] - starts[t]) for t in range(T))
-    return BatchCounts(T, batch, tuple(int(d) for d in dims), elem_bytes, idx_bytes, weighted, per)
+    if batch > 0:
+        lens = (offsets[1:T * batch + 1] - offsets[:T * batch]).view(T, batch)
+        nonempty = tuple(int(x) for x in (lens > 0).sum(1).to("cpu").tolist())
+    else:
+        nonempty = (0,) * T
+    return BatchCounts(T, batch, tuple(int(d) for d in dims), elem_bytes, idx_bytes, weighted, per,
+                       nonempty)
 
 
 def forward_bytes(c: BatchCounts) -> dict[str, int]:
@@ -125,7 +132,7 @@ def radix_passes(rows) -> int:
     """8-bit passes over the row number of the largest table (ranges sorted per table)."""
     largest = max(1, int(max(rows)))
     bits = 1
-    while bits < 32 and (1 << bits) < largest:
+    while bits < 32 and (1 << bits) <= largest:  # keys 0 .. rows_t (rows_t: out of range)
         bits += 1
     return (bits + 7) // 8
 
@@ -144,6 +151,22 @@ def component_bytes(c: BatchCounts, unique_per_table, rows, packed: bool) -> dic
         "bwd.rle": 8 * n + 8 * U,
         "bwd.reduce": b["grad_gather"] + 4 * n + (8 * n if packed else 0) + 4 * U + b["grads"]
         + 16 * U,
+    }
+
+
+def component_compulsory_bytes(c: BatchCounts, unique_per_table, packed: bool) -> dict[str, int]:
+    """Compulsory bytes of the two gather kernels: what they must move even when
+    every repeated row comes from cache, i.e. each distinct table row (forward)
+    or each non-empty bag's grad_out slice (backward reduce) once, plus their
+    per-lookup and per-row streams and outputs. With the L2 flushed before a
+    step this is the least DRAM traffic of the launch."""
+    U = int(sum(int(u) for u in unique_per_table))
+    n = c.n
+    slices = sum(int(k) * d * 4 for k, d in zip(c.nonempty_per_table, c.dims))
+    grads = sum(int(u) * d * 4 for u, d in zip(unique_per_table, c.dims))
+    return {
+        "fwd.gather": forward_unique_bytes(c, unique_per_table),
+        "bwd.reduce": slices + 4 * n + (8 * n if packed else 0) + 4 * U + grads + 16 * U,
     }
 
 

@@ -33,7 +33,7 @@ EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
            "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad",
            "cb_tbe_backward_apply", "cb_tbe_apply_sparse", "cb_kjt_replicate",
-           "cb_tbe_sorted_payloads")
+           "cb_tbe_sorted_payloads", "cb_gather_ceiling")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -89,12 +89,13 @@ def load_library() -> ctypes.CDLL:
                                         ctypes.c_float, p, p]
     lib.cb_kjt_replicate.argtypes = [p, p, p, ctypes.c_int, i32, i32, i64, i32, p, p, p, p]
     lib.cb_tbe_sorted_payloads.argtypes = [p, p, i64, p]
+    lib.cb_gather_ceiling.argtypes = [p, i64, i32, p, i64, p, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
                  "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward",
                  "cb_tbe_weight_grad", "cb_tbe_backward_apply", "cb_kjt_replicate",
-                 "cb_tbe_sorted_payloads"):
+                 "cb_tbe_sorted_payloads", "cb_gather_ceiling"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -410,6 +411,27 @@ def fm_backward(y: torch.Tensor, grad_fm: torch.Tensor, num_fields: int,
         stream = ctypes.c_void_p(torch.cuda.current_stream(y.device).cuda_stream)
         _check(lib.cb_fm_backward(_ptr(y), _ptr(grad_fm), B, num_fields, D, stride, _ptr(out),
                                   stream), "cb_fm_backward")
+    return out
+
+
+# ----------------------------------------------------------------------------- measurement aid
+
+def gather_ceiling(rows: torch.Tensor, indices: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+    """Random-row gather out of `rows` ([R, row_bytes / 4] fp32, L2-sized) at `indices`
+    (int32 viewed as uint32) with the walkers' load shape (cb_gather_ceiling); returns
+    the per-32-item sums."""
+    lib = load_library()
+    if rows.device.type != "cuda" or rows.dtype != torch.float32 or rows.dim() != 2 or not rows.is_contiguous():
+        raise ValueError("rows must be a contiguous 2-D fp32 CUDA tensor")
+    if indices.device != rows.device or indices.dtype != torch.int32:
+        raise ValueError("indices must be int32 on the device of rows")
+    n = indices.numel()
+    if out is None:
+        out = torch.empty(max((n + 31) // 32, 1), dtype=torch.float32, device=rows.device)
+    with torch.cuda.device(rows.device):
+        stream = ctypes.c_void_p(torch.cuda.current_stream(rows.device).cuda_stream)
+        _check(lib.cb_gather_ceiling(_ptr(rows), rows.shape[0], rows.shape[1] * 4, _ptr(indices.contiguous()),
+                                     n, _ptr(out), stream), "cb_gather_ceiling")
     return out
 
 

@@ -13,7 +13,7 @@ def _declared_functions():
     with open(os.path.join(ROOT, "include", "cb_tbe.h")) as f:
         text = f.read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(cb_(?:tbe|fm|kjt)_\w+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(cb_(?:tbe|fm|kjt|gather)_\w+)\s*\(", text)))
 
 
 @pytest.fixture(scope="module")
@@ -110,3 +110,14 @@ def test_create_refuses_a_key_space_beyond_32_bits(lib):
     h = ctypes.c_void_p()
     descs = (tbe.CbTableDesc * 2)(tbe.CbTableDesc(4096, 2**31, 4, 0), tbe.CbTableDesc(4096, 2**31 - 2, 4, 0))
     assert lib.cb_tbe_create(descs, 2, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
+
+
+def test_gather_ceiling_rejects_bad_sizes_on_the_host(lib):
+    from paper_2609_30656_gb300 import tbe
+    p = ctypes.c_void_p
+    f = lib.cb_gather_ceiling
+    assert f(p(4096), 100, 96, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # row size
+    assert f(p(4100), 100, 512, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # alignment
+    assert f(p(4096), 0, 512, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # no rows
+    assert f(p(4096), 100, 512, None, 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # no indices
+    assert f(p(4096), 100, 512, None, 0, None, None) == tbe.CB_OK  # nothing to do

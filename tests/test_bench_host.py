@@ -27,6 +27,20 @@ def test_forward_and_backward_bytes_by_hand():
     assert metrics.forward_unique_bytes(c, [3, 1]) == f["total"] - f["rows"] + 3 * 8 + 1 * 16
 
 
+def test_compulsory_bytes_by_hand():
+    # 2 tables (dims 4 and 8, fp16), batch 3: table 0 has bags of 2, 0, 3 lookups,
+    # table 1 bags of 1, 1, 0 -> 2 and 2 non-empty bags; 3 and 1 distinct rows
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts((4, 8), 2, 3, off, weighted=False)
+    assert c.nonempty_per_table == (2, 2)
+    cb = metrics.component_compulsory_bytes(c, [3, 1], packed=False)
+    assert cb["fwd.gather"] == metrics.forward_unique_bytes(c, [3, 1])
+    slices = 2 * 4 * 4 + 2 * 8 * 4
+    grads = 3 * 4 * 4 + 1 * 8 * 4
+    assert cb["bwd.reduce"] == slices + 4 * 7 + 4 * 4 + grads + 16 * 4
+    assert metrics.component_compulsory_bytes(c, [3, 1], packed=True)["bwd.reduce"] == cb["bwd.reduce"] + 8 * 7
+
+
 def test_weight_grad_bytes_by_hand():
     # 2 tables (dims 4 and 8, fp16), batch 3, lookups 5 and 2
     off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
@@ -63,7 +77,9 @@ def test_fm_bytes_by_hand():
 
 
 def test_radix_passes_follow_row_bits():
-    assert metrics.radix_passes([256]) == 1
+    # keys 0 .. rows_t (the spare key rows_t marks an out-of-range lookup)
+    assert metrics.radix_passes([255]) == 1
+    assert metrics.radix_passes([256]) == 2
     assert metrics.radix_passes([257]) == 2
     assert metrics.radix_passes([5_000_000] * 100) == 3   # 23-bit rows, per-table ranges
     assert metrics.radix_passes([100_000] * 8) == 3       # 17-bit rows
@@ -139,7 +155,7 @@ def test_report_written_from_measured_components(tmp_path):
     c = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, off, weighted=False)
     comp_ms = {"fwd.prep": 0.01, "fwd.gather": 1.0, "fwd.fixup": 0.01, "bwd.keygen": 0.2,
                "bwd.sort": 0.5, "bwd.rle": 0.1, "bwd.reduce": 2.0}
-    comp_bytes = {"fwd.gather": 3 * 6e9, "bwd.reduce": 3 * 8e9}  # over the 3 timed steps
+    comp_bytes = {"fwd.gather": 6e9, "bwd.reduce": 8e9}  # per step (the breakdown run's mean)
     line = {"steps": 3, "ms_per_step": 4.0, "config": {"workload": "tiny"},
             "next_rows": {"fm": {"forward": {"ms": 0.1, "bytes": 1e6}, "backward": {"ms": 0.2, "bytes": 2e6}},
                           "weight_grad": {"ms": 0.3, "bytes": 3e6},
@@ -158,3 +174,35 @@ def test_report_written_from_measured_components(tmp_path):
     # the step's rate covers its own kernels: (6 + 8) GB over their 3.82 ms
     assert step["est_avg_bw_gbs"] == pytest.approx(14e9 / 3.82e-3 / 1e9, abs=0.1)
     assert "| fwd.gather |" in (tmp_path / "r.md").read_text().replace("&nbsp;", "")
+
+
+def test_quantiles_and_timing_summary():
+    xs = [5.0, 1.0, 3.0, 2.0, 4.0]
+    assert bench.quantile(xs, 0.5) == 3.0
+    assert bench.quantile(xs, 0.1) == pytest.approx(1.4)
+    assert bench.quantile(xs, 0.9) == pytest.approx(4.6)
+    s = bench.timing_summary(xs)
+    assert s["median"] == 3.0 and s["p10"] == 1.4 and s["p90"] == 4.6 and s["samples"] == 5
+
+
+def test_roofline_uses_dram_traffic_when_recorded(monkeypatch):
+    w = wl.scaled(wl.get_workload("cfg5"), num_tables=2, batch=3, rows=10)
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, off, weighted=False)
+    comp_ms = {"fwd.gather": 1.0, "bwd.reduce": 2.0}
+    comp_bytes = {"fwd.gather": 6e9, "bwd.reduce": 40e9}  # 20 TB/s of every-lookup bytes
+    comp_compulsory = {"fwd.gather": 1e9, "bwd.reduce": 4e9}
+    monkeypatch.setattr(bench, "recorded_traffic", lambda k, wl_: None)
+    r = bench.roofline_of("x", comp_ms, comp_bytes, comp_compulsory, 5000.0, "measured", None, [c], w)
+    assert r["kernel"] == "bwd.reduce" and r["basis"] == "compulsory"
+    assert r["achieved"] == pytest.approx(2000.0) and r["frac"] == pytest.approx(0.4)
+    assert r["alg_frac"] == pytest.approx(4.0)  # the reuse-inflated figure under its own name
+    monkeypatch.setattr(bench, "recorded_traffic", lambda k, wl_: 6e9)
+    r = bench.roofline_of("x", comp_ms, comp_bytes, comp_compulsory, 5000.0, "measured", None, [c], w)
+    assert r["basis"] == "dram" and r["frac"] == pytest.approx(0.6) and r["traffic"] == 6e9
+    ceiling = {"512": {"gbs": 20000.0}, "256": {"gbs": 20000.0}}
+    r = bench.roofline_of("x", comp_ms, comp_bytes, comp_compulsory, 5000.0, "measured", ceiling, [c], w)
+    gathered = metrics.backward_bytes(c, [0, 0])["grad_gather"]
+    assert r["l2_gather_gbs"] == round(gathered / 2e-3 / 1e9, 1)
+    assert r["frac_l2"] == pytest.approx(gathered / 2e-3 / 1e9 / 20000.0, abs=1e-4)
+    assert r["l2_ceiling_row_bytes"] == 512  # fp32 grad_out slices of dim 128
