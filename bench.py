@@ -486,8 +486,10 @@ def roofline_of(workload, comp_ms, comp_bytes, comp_compulsory, peak, peak_kind,
     traffic = recorded_traffic(dominant, workload)
     if traffic:
         achieved, basis = traffic / t / 1e9, "dram"
-    else:
+    elif comp:
         achieved, basis = comp / t / 1e9, "compulsory"
+    else:  # a streaming kernel without reuse: its algorithmic bytes are compulsory
+        achieved, basis = alg / t / 1e9, "algorithmic"
     r = {"bound": "hbm", "kernel": dominant, "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
          "frac": round(achieved / peak, 4), "basis": basis,
          "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"

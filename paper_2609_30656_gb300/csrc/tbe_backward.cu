@@ -506,39 +506,71 @@ namespace cbtbe {
 // loads before any store. Lane l owns columns 4l + 128m, m < M (the fused
 // step's order, so both give the same sums of squares). Nothing is done when
 // the gradient buffers were too small (the backward then wrote no rows).
+#ifndef CB_APPLY_MIN_BLOCKS
+#define CB_APPLY_MIN_BLOCKS 3  // resident blocks per SM for rows of up to 128 columns (wider: 2)
+#endif
+#ifndef CB_APPLY_ROWS_M1
+#define CB_APPLY_ROWS_M1 2  // rows stepped at once for rows of up to 128 columns
+#endif
+constexpr int kApplyShTables = 1024;  // table offsets staged in shared memory up to this many tables
+
+// One lane's row of a group of 32: where its stored row, gradient and state
+// are, its (dim, dtype), and its previous Adagrad state.
+struct ApplyRow {
+    unsigned long long row;    // start of the stored row
+    unsigned long long grad;   // start of its gradient
+    unsigned long long state;  // its state word (Adagrad), or 0
+    int shape;                 // dim << 2 | dtype (dim 0: nothing loaded or stored)
+    float m0;
+};
+
+__device__ __forceinline__ ApplyRow apply_row_meta(const Problem& P, const BwdOut& O, const int64_t* toff,
+                                                   int64_t u0, int64_t U, int64_t F, int lane, bool adagrad) {
+    const int64_t u = min64(u0 + lane, U - 1);
+    const int64_t id = __ldg(O.unique_ids + u);
+    const int64_t goff = __ldg(O.grad_offsets + u);
+    int lo = 0, hi = P.T;  // table_offsets[lo] <= u < table_offsets[lo + 1]
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (toff[mid] <= u) lo = mid;
+        else hi = mid;
+    }
+    const TableDev& td = P.tables[lo];
+    const int64_t row = id - td.row_base;
+    // A gradient this handle's backward wrote always passes; a row that does not
+    // (buffers from elsewhere) is skipped and reported, never followed outside
+    // a table, the gradient or the state.
+    const bool ok = row >= 0 && row < td.rows && goff >= 0 && goff + td.dim <= F;
+    if (!ok && u0 + lane < U) set_error(P.error, CB_ERR_INDEX_OOB);
+    ApplyRow m;
+    m.row = reinterpret_cast<unsigned long long>(row_ptr(td, ok ? row : 0));
+    m.grad = reinterpret_cast<unsigned long long>(O.grads + (ok ? goff : 0));
+    m.state = adagrad && ok ? reinterpret_cast<unsigned long long>(O.state[lo] + row) : 0ull;
+    m.shape = ((ok ? td.dim : 0) << 2) | td.dtype;
+    m.m0 = m.state ? *reinterpret_cast<const float*>(m.state) : 0.f;
+    return m;
+}
+
 template <int M, int R>
-__global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid_constant__ Problem P,
-                                                                    const __grid_constant__ BwdOut O) {
+__global__ void __launch_bounds__(kWarpThreads, M == 1 ? CB_APPLY_MIN_BLOCKS : 2)
+    apply_sparse_kernel(const __grid_constant__ Problem P, const __grid_constant__ BwdOut O) {
     static_assert(32 % R == 0, "rows per step divide the warp's 32");
+    // The per-table first rows, for the bisection that finds each row's table.
+    __shared__ int64_t sh_toff[kApplyShTables + 1];
+    const bool staged = P.T <= kApplyShTables;
+    if (staged)
+        for (int t = threadIdx.x; t <= P.T; t += blockDim.x) sh_toff[t] = __ldg(O.table_offsets + t);
+    __syncthreads();
+    const int64_t* toff = staged ? sh_toff : O.table_offsets;
     const int lane = threadIdx.x & 31;
     const int64_t U = *O.num_unique;
     const int64_t F = *O.num_floats;
     if (U > O.cap_rows || F > O.cap_floats) return;
     const bool adagrad = O.apply == kApplyAdagrad;
+    // (Loading the next group's ids, offsets and states while this group steps
+    // was measured: no faster on cfg5.)
     for (int64_t u0 = warp_id_global() * 32; u0 < U; u0 += warps_in_grid() * 32) {
-        // this lane's row: start of its stored row, of its gradient and state
-        const int64_t u = min64(u0 + lane, U - 1);
-        const int64_t id = __ldg(O.unique_ids + u);
-        const int64_t goff = __ldg(O.grad_offsets + u);
-        int lo = 0, hi = P.T;  // table_offsets[lo] <= u < table_offsets[lo + 1]
-        while (hi - lo > 1) {
-            const int mid = (lo + hi) >> 1;
-            if (__ldg(O.table_offsets + mid) <= u) lo = mid;
-            else hi = mid;
-        }
-        const TableDev& td = P.tables[lo];
-        const int64_t row = id - td.row_base;
-        // A gradient this handle's backward wrote always passes; a row that
-        // does not (buffers from elsewhere) is skipped and reported, never
-        // followed outside a table, the gradient or the state.
-        const bool ok = row >= 0 && row < td.rows && goff >= 0 && goff + td.dim <= F;
-        if (!ok && u0 + lane < U) set_error(P.error, CB_ERR_INDEX_OOB);
-        const unsigned long long my_row = reinterpret_cast<unsigned long long>(row_ptr(td, ok ? row : 0));
-        const unsigned long long my_grad = reinterpret_cast<unsigned long long>(O.grads + (ok ? goff : 0));
-        const unsigned long long my_state =
-            adagrad && ok ? reinterpret_cast<unsigned long long>(O.state[lo] + row) : 0ull;
-        const int my_shape = ((ok ? td.dim : 0) << 2) | td.dtype;  // dim 0: nothing loaded or stored
-        const float my_m0 = my_state ? *reinterpret_cast<const float*>(my_state) : 0.f;
+        const ApplyRow cur = apply_row_meta(P, O, toff, u0, U, F, lane, adagrad);
         const int rows_here = static_cast<int>(min64(32, U - u0));
         for (int r0 = 0; r0 < rows_here; r0 += R) {
             char* rp[R];
@@ -547,9 +579,9 @@ __global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid
             uint4 x[R][M];
 #pragma unroll
             for (int i = 0; i < R; ++i) {
-                rp[i] = reinterpret_cast<char*>(__shfl_sync(kFull, my_row, r0 + i));
-                const float* gp = reinterpret_cast<const float*>(__shfl_sync(kFull, my_grad, r0 + i));
-                shape[i] = __shfl_sync(kFull, my_shape, r0 + i);
+                rp[i] = reinterpret_cast<char*>(__shfl_sync(kFull, cur.row, r0 + i));
+                const float* gp = reinterpret_cast<const float*>(__shfl_sync(kFull, cur.grad, r0 + i));
+                shape[i] = __shfl_sync(kFull, cur.shape, r0 + i);
 #pragma unroll
                 for (int m = 0; m < M; ++m) {
                     const int x0 = lane * 4 + 128 * m;
@@ -583,9 +615,9 @@ __global__ void __launch_bounds__(kWarpThreads) apply_sparse_kernel(const __grid
                 for (int i = 0; i < R; ++i)
                     if (lane == r0 + i) mine = sq[i];
                 float my_scale = O.lr;
-                if (lane >= r0 && lane < r0 + R && lane < rows_here && my_state) {
-                    const float m = my_m0 + mine / static_cast<float>(my_shape >> 2);
-                    *reinterpret_cast<float*>(my_state) = m;
+                if (lane >= r0 && lane < r0 + R && lane < rows_here && cur.state) {
+                    const float m = cur.m0 + mine / static_cast<float>(cur.shape >> 2);
+                    *reinterpret_cast<float*>(cur.state) = m;
                     my_scale = O.lr / (sqrtf(m) + O.eps);
                 }
 #pragma unroll
@@ -612,7 +644,7 @@ void launch_apply_sparse_m(const Problem& P, const BwdOut& O, int num_sms, cudaS
 }
 
 void launch_apply_sparse(const Problem& P, const BwdOut& O, int num_sms, cudaStream_t s) {
-    if (P.dmax <= 128) launch_apply_sparse_m<1, 8>(P, O, num_sms, s);
+    if (P.dmax <= 128) launch_apply_sparse_m<1, CB_APPLY_ROWS_M1>(P, O, num_sms, s);
     else if (P.dmax <= 256) launch_apply_sparse_m<2, 4>(P, O, num_sms, s);
     else launch_apply_sparse_m<4, 2>(P, O, num_sms, s);
 }

@@ -110,6 +110,23 @@ struct FwdPolicy {
     }
 };
 
+// Groups of row loads kept in flight per warp through shared memory by the
+// row walker (0: loads into registers).
+#ifndef CB_GATHER_ASYNC
+#define CB_GATHER_ASYNC 0
+#endif
+constexpr int kGatherAsync = CB_GATHER_ASYNC;
+
+// 16-byte slots per lane of a warp's ring: (groups in flight + 1) load groups.
+template <class Pol, int GC>
+__host__ __device__ constexpr int gather_ring_slots() {
+    constexpr int steps = GC > 0 ? 32 / GC : 1;
+    constexpr int ug = Pol::kUnroll < steps ? Pol::kUnroll : steps;
+    constexpr int groups = steps / ug;  // load groups per batch of 32 items
+    constexpr int depth = kGatherAsync < groups ? kGatherAsync : groups;
+    return kGatherAsync > 0 ? (depth + 1) * ug : 0;
+}
+
 template <int DT, int VPL, bool WEIGHTED, int GC>
 __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
     fwd_gather_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q, void* out,
@@ -141,7 +158,14 @@ __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
         if (lane == 0) Q.tail_owner[j] = -1;
         if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
             __shared__ EndSlot slots[kWarpThreads / 32][32];
-            walk_rows<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+            if constexpr (kGatherAsync > 0) {
+                extern __shared__ __align__(16) uint4 ring[];
+                constexpr int kSlots = gather_ring_slots<FwdPolicy<DT, VPL, WEIGHTED>, GC>();
+                walk_rows<FwdPolicy<DT, VPL, WEIGHTED>, GC, kGatherAsync>(
+                    pol, c, P.zero_row, lane, slots[threadIdx.x >> 5], ring + (threadIdx.x >> 5) * kSlots * 32);
+            } else {
+                walk_rows<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+            }
         } else {
             walk_chunk<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane);
         }
@@ -149,12 +173,24 @@ __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
     }
 }
 
+// Dynamic shared memory of the gather: the warps' rings of staged row loads.
+template <int DT, int VPL, bool W, int GC>
+static size_t gather_smem() {
+    if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER)
+        return sizeof(uint4) * 32 * (kWarpThreads / 32) * gather_ring_slots<FwdPolicy<DT, VPL, W>, GC>();
+    return 0;
+}
+
 template <int DT, int VPL, bool W, int GC>
 static int gather_grid(int num_sms) {
     static int per_sm = -1;
     if (per_sm < 0) {
+        const size_t smem = gather_smem<DT, VPL, W, GC>();
+        if (smem > 0)
+            cudaFuncSetAttribute(fwd_gather_kernel<DT, VPL, W, GC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem));
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fwd_gather_kernel<DT, VPL, W, GC>,
-                                                          kWarpThreads, 0) != cudaSuccess ||
+                                                          kWarpThreads, smem) != cudaSuccess ||
             per_sm < 1)
             per_sm = 1;
     }
@@ -167,10 +203,12 @@ static void launch_gather_layout(const Problem& P, const Plan& Q, void* out, int
     const int64_t need = (chunk_bound + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
     if (P.weights) {
         const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL, true, GC>(num_sms)));
-        fwd_gather_kernel<DT, VPL, true, GC><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
+        fwd_gather_kernel<DT, VPL, true, GC><<<max(grid, 1), kWarpThreads, gather_smem<DT, VPL, true, GC>(), s>>>(
+            P, Q, out, cls);
     } else {
         const int grid = static_cast<int>(min64(need, gather_grid<DT, VPL, false, GC>(num_sms)));
-        fwd_gather_kernel<DT, VPL, false, GC><<<max(grid, 1), kWarpThreads, 0, s>>>(P, Q, out, cls);
+        fwd_gather_kernel<DT, VPL, false, GC><<<max(grid, 1), kWarpThreads, gather_smem<DT, VPL, false, GC>(), s>>>(
+            P, Q, out, cls);
     }
 }
 

@@ -282,6 +282,8 @@ __host__ __device__ __forceinline__ int dtype_bytes(int dtype) { return dtype ==
 // acc += w * row (WEIGHTED) or acc += row. Half-precision rows use the
 // mixed-precision add of sm_100+ (f16/bf16 operand widened exactly, fp32 sum),
 // which is the same arithmetic as widening first and then adding.
+// (Measured on cfg5: widening fp16 pairs first and adding in fp32 took 29 %
+// more instructions and 11 % more time.)
 template <int DT, bool WEIGHTED>
 __device__ __forceinline__ void accumulate(float (&a)[Storage<DT>::kElems], const uint4& x, float w) {
     const uint32_t word[4] = {x.x, x.y, x.z, x.w};
@@ -555,9 +557,30 @@ struct EndSlot {
     int32_t len;  // segment length, or -1 when it began in an earlier chunk
 };
 
-template <class Pol, int G>
+// Loads of rows staged in shared memory (D > 0): each group of UG row steps is
+// copied with cp.async into a per-warp ring of D + 1 groups of slots (16 bytes
+// per lane and step), D groups ahead of the one being added, so that D * UG
+// steps of rows are in flight per warp without holding registers. A slot is
+// refilled one group after it was read, when its values have been added. The
+// decoded payloads of the next batch are kept for the prefetch across the
+// batch boundary. D = 0: the rows are loaded into registers one group at a
+// time.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 16;\n" ::"r"(
+                     static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
+template <class Pol, int G, int D = 0>
 __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uint4* zero_row,
-                                          int lane, EndSlot* slots) {
+                                          int lane, EndSlot* slots, uint4* ring = nullptr) {
     static_assert(G == 1 || G == 2 || G == 4 || G == 8, "rows per warp step");
     static_assert(Pol::kVpl == 1, "one vector per lane");
     constexpr int E = Pol::kElems;
@@ -589,6 +612,7 @@ __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uin
     int32_t s_cur = seg < c.seg_hi ? rel_pos(pol.seg_begin(seg), c.k0) : kRelHi;
     int32_t my_end = seg + lane < c.seg_hi ? rel_pos(pol.seg_end(seg + lane), c.k0) : kRelHi;
     uint32_t mask = 0;
+    int ce_async = 0;  // next entry of the segment-end list (staged loads)
 
     // Segments ending at or before `bend` (the batch starts at `base`) leave the
     // window: non-empty ones are listed and marked in `mask`, empty ones owned
@@ -695,6 +719,110 @@ __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uin
             }
         }
     };
+
+    if constexpr (D > 0) {
+        constexpr int kGroups = 32 / kGroupItems;  // load groups per batch
+        // groups in flight: at most a batch's, so the prefetch reaches at most
+        // one batch ahead
+        constexpr int DD = D < kGroups ? D : kGroups;
+        constexpr int kRing = DD + 1;              // groups of slots in the ring
+        // The rows of load group q (0 .. kGroups-1) of a batch whose decoded
+        // row numbers are `aa` and first position `bbase` go to ring group `rg`.
+        auto issue = [&](int rg, uint32_t aa, int q, int32_t bbase) {
+#pragma unroll
+            for (int u = 0; u < UG; ++u) {
+                const int src = q * kGroupItems + u * G + g;
+                const uint32_t a = __shfl_sync(kFull, aa, src);
+                const char* p = (a != kInvalid && bbase + src < len)
+                                    ? lane_base + static_cast<uint64_t>(a) * row_bytes
+                                    : reinterpret_cast<const char*>(zrow);
+                cp_async16(ring + (rg * UG + u) * 32 + lane, p);
+            }
+            cp_async_commit();
+        };
+        // Decoded payloads of this batch and the next; raw payloads two ahead.
+        uint32_t a0 = kInvalid, a1 = kInvalid;
+        float w0 = 0.f, w1 = 0.f;
+        typename Pol::Raw raw = Pol::none();
+        if (lane < len) raw = pol.fetch(c.k0 + lane);
+        if (lane < len) pol.decode(raw, a0, w0);
+        raw = Pol::none();
+        if (32 + lane < len) raw = pol.fetch(c.k0 + 32 + lane);
+#pragma unroll
+        for (int q = 0; q < DD; ++q) issue(q, a0, q, 0);
+        int rd = 0;  // ring group read next
+        for (int32_t base = 0; base < len; base += 32) {
+            const int nb = min(32, len - base);
+            a1 = kInvalid;
+            w1 = 0.f;
+            if (base + 32 + lane < len) pol.decode(raw, a1, w1);
+            raw = Pol::none();
+            if (base + 64 + lane < len) raw = pol.fetch(c.k0 + base + 64 + lane);
+            scan(base, base + nb);
+            for (int q = 0; q < kGroups; ++q) {
+                if (base + q * kGroupItems >= len) {
+                    // past the chunk: the groups still in flight carry zeros
+                    continue;
+                }
+                cp_async_wait<DD - 1>();
+                uint4 buf[UG];
+                float wt[UG];
+#pragma unroll
+                for (int u = 0; u < UG; ++u) {
+                    buf[u] = ring[(rd * UG + u) * 32 + lane];
+                    wt[u] = W ? __shfl_sync(kFull, w0, q * kGroupItems + u * G + g) : 1.f;
+                }
+                // refill the ring group read one group ago with group q + DD
+                const int wr = rd == 0 ? kRing - 1 : rd - 1;
+                if (q + DD < kGroups) issue(wr, a0, q + DD, base);
+                else issue(wr, a1, q + DD - kGroups, base + 32);
+                rd = rd + 1 == kRing ? 0 : rd + 1;
+                const uint32_t m = (mask >> (q * kGroupItems)) & kGroupMask;
+                if (m == 0) {
+#pragma unroll
+                    for (int u = 0; u < UG; ++u) accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                    continue;
+                }
+#pragma unroll
+                for (int u = 0; u < UG; ++u) {
+                    uint32_t mu = (m >> (u * G)) & kStepMask;
+                    if (mu == 0) {
+                        accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                        continue;
+                    }
+                    bool added = false;
+                    do {
+                        const int p = __ffs(mu) - 1;
+                        if (!added && g <= p) {
+                            accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                            added = true;
+                        }
+                        flush(slots[ce_async++], true);
+                        mu &= mu - 1;
+                    } while (mu);
+                    if (!added) accumulate<Pol::kDtype, W>(ain, buf[u], wt[u]);
+                }
+            }
+            ce_async = 0;
+            if (kTwoLevel) {
+#pragma unroll
+                for (int x = 0; x < E; ++x) {
+                    aout[x] += ain[x];
+                    ain[x] = 0.f;
+                }
+            }
+            a0 = a1;
+            w0 = w1;
+        }
+        cp_async_wait_all();
+        __syncwarp();
+        scan(len, len);
+        if (seg < c.seg_hi && s_cur < len) {
+            if (s_cur >= 0 && lane == 0) pol.seg_meta(seg);
+            flush(EndSlot{seg, s_cur >= 0 ? 0 : -1}, false);
+        }
+        return;
+    }
 
     typename Pol::Raw nxt = Pol::none();
     if (lane < len) nxt = pol.fetch(c.k0 + lane);

@@ -71,38 +71,63 @@ __device__ __forceinline__ uint32_t shared_add_if(uint32_t* p, uint32_t v, bool 
 // counter of that digit and shares the old value. A warp's shared-memory
 // atomics take effect in issue order, so item j's lanes count before item
 // j + 1's, and lanes of one item by lane: the rank follows the position.
-// Positions past the tile count under the extra digit kRadix.
+// Positions past the tile count under the extra digit kRadix. The matches of
+// kRankBatch items are found before their atomics are issued (in item order),
+// so that independent match, atomic and shuffle latencies overlap.
+#ifndef CB_RANK_BATCH
+#define CB_RANK_BATCH 2
+#endif
+constexpr int kRankBatch = CB_RANK_BATCH;
+static_assert(kSortItems % kRankBatch == 0, "rank batches divide the items");
+
 __device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int tile_count, uint32_t key_base,
                                           int shift, uint32_t (*sh_warp)[kRadix + 1],
                                           uint32_t (&rank2)[kSortItems / 2]) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const uint32_t lt_mask = (1u << lane) - 1u;
 #pragma unroll
-    for (int j = 0; j < kSortItems; ++j) {
-        const int local = wid * (32 * kSortItems) + j * 32 + lane;
-        const uint32_t d = local < tile_count ? sort_digit(key[j], key_base, shift) : kRadix;
-        const uint32_t peers = __match_any_sync(kFull, d);
-        const int leader = __ffs(peers) - 1;
-        const uint32_t before =
-            shared_add_if(&sh_warp[wid][d], static_cast<uint32_t>(__popc(peers)), lane == leader);
-        const uint32_t r = __shfl_sync(kFull, before, leader) + __popc(peers & lt_mask);
-        if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;  // two 16-bit ranks per register
+    for (int j0 = 0; j0 < kSortItems; j0 += kRankBatch) {
+        uint32_t d[kRankBatch], peers[kRankBatch], before[kRankBatch];
+#pragma unroll
+        for (int i = 0; i < kRankBatch; ++i) {
+            const int j = j0 + i;
+            const int local = wid * (32 * kSortItems) + j * 32 + lane;
+            d[i] = local < tile_count ? sort_digit(key[j], key_base, shift) : kRadix;
+            peers[i] = __match_any_sync(kFull, d[i]);
+        }
+#pragma unroll
+        for (int i = 0; i < kRankBatch; ++i) {
+            const int leader = __ffs(peers[i]) - 1;
+            before[i] = shared_add_if(&sh_warp[wid][d[i]], static_cast<uint32_t>(__popc(peers[i])), lane == leader);
+        }
+#pragma unroll
+        for (int i = 0; i < kRankBatch; ++i) {
+            const int j = j0 + i;
+            const int leader = __ffs(peers[i]) - 1;
+            const uint32_t r = __shfl_sync(kFull, before[i], leader) + __popc(peers[i] & lt_mask);
+            if (j & 1) rank2[j >> 1] |= r << 16; else rank2[j >> 1] = r;  // two 16-bit ranks per register
+        }
     }
 }
 
-// The tile laid out by digit in shared memory (slot = the digit's tile-local
-// start + the warp's prefix + the rank): every slot first (the counters are
-// read-only here), then the stores.
+// The tile laid out by digit in shared memory (slot = the warp's start of the
+// digit, which holds the digit's tile-local start plus the counts of earlier
+// warps, + the rank): every slot first (the counters are read-only here), then
+// the stores. With CB_SORT_KV_PAIRS each (key, payload) pair goes to shared
+// memory as one 8-byte word.
+#ifndef CB_SORT_KV_PAIRS
+#define CB_SORT_KV_PAIRS 0
+#endif
 __device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], const uint32_t (&val)[kSortItems],
                                              uint32_t (&rank2)[kSortItems / 2], int tile_count, uint32_t key_base,
                                              int shift, const uint32_t (*sh_warp)[kRadix + 1],
-                                             const uint32_t* sh_start, uint32_t* sh_keys, uint32_t* sh_vals) {
+                                             uint32_t* sh_keys, uint32_t* sh_vals) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
     for (int j = 0; j < kSortItems; ++j) {
         const uint32_t dd = sort_digit(key[j], key_base, shift);
         const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
-        const uint32_t pos = (sh_start[dd] + sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
+        const uint32_t pos = (sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
         rank2[j >> 1] = (j & 1) ? ((rank2[j >> 1] & 0xffffu) | (pos << 16))
                                 : ((rank2[j >> 1] & 0xffff0000u) | pos);
     }
@@ -111,8 +136,12 @@ __device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], 
         const int local = wid * (32 * kSortItems) + j * 32 + lane;
         if (local < tile_count) {
             const uint32_t pos = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
-            sh_keys[pos] = key[j];
-            sh_vals[pos] = val[j];
+            if (CB_SORT_KV_PAIRS) {
+                reinterpret_cast<uint2*>(sh_keys)[pos] = make_uint2(key[j], val[j]);
+            } else {
+                sh_keys[pos] = key[j];
+                sh_vals[pos] = val[j];
+            }
         }
     }
 }
@@ -132,8 +161,14 @@ __device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, ui
 #pragma unroll
         for (int j = 0; j < kHalf; ++j) {
             const int i = tid + (h * kHalf + j) * kSortThreads;
-            key[j] = i < tile_count ? sh_keys[i] : 0u;
-            val[j] = i < tile_count ? sh_vals[i] : 0u;
+            if (CB_SORT_KV_PAIRS) {
+                const uint2 kv = i < tile_count ? reinterpret_cast<const uint2*>(sh_keys)[i] : make_uint2(0u, 0u);
+                key[j] = kv.x;
+                val[j] = kv.y;
+            } else {
+                key[j] = i < tile_count ? sh_keys[i] : 0u;
+                val[j] = i < tile_count ? sh_vals[i] : 0u;
+            }
         }
 #pragma unroll
         for (int j = 0; j < kHalf; ++j)
@@ -155,7 +190,6 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     uint32_t* sh_vals = sh_dyn + kSortTile;                // tile-sorted payloads
     __shared__ uint32_t sh_warp[kSortWarps][kRadix + 1];   // per-warp counts, then prefixes
                                                            // (slot kRadix: positions past the tile)
-    __shared__ uint32_t sh_start[kRadix];                  // tile-local start of each digit
     __shared__ int32_t sh_goff[kRadix];                    // global destination - local index
     __shared__ int64_t sh_scan[33];
     __shared__ uint32_t sh_tile;
@@ -204,7 +238,8 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
     store_volatile(my_status, (tile == first_tile ? kFlagIncl : kFlagAgg) | count);
     int64_t total;
     const int64_t start = block_excl_scan(count, sh_scan, &total);
-    sh_start[d] = static_cast<uint32_t>(start);
+#pragma unroll
+    for (int w = 0; w < kSortWarps; ++w) sh_warp[w][d] += static_cast<uint32_t>(start);
 
     // Decoupled look-back over earlier tiles for digit d, kLookbackWindow
     // predecessors per round (independent loads), bounded in time.
@@ -263,7 +298,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         static_cast<int64_t>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) + excl - start);
     __syncthreads();
 
-    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
+    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_keys, sh_vals);
     __syncthreads();
     if (sh_abort) return;
     write_tile(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
@@ -370,7 +405,6 @@ __global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const So
     uint32_t* sh_vals = sh_dyn + kSortTile;                // tile-sorted payloads
     __shared__ uint32_t sh_warp[kSortWarps][kRadix + 1];   // per-warp counts, then prefixes
                                                            // (slot kRadix: positions past the tile)
-    __shared__ uint32_t sh_start[kRadix];                  // tile-local start of each digit
     __shared__ int32_t sh_goff[kRadix];                    // global destination - local index
     __shared__ int64_t sh_scan[33];
 
@@ -405,10 +439,11 @@ __global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const So
     }
     int64_t total;
     const int64_t start = block_excl_scan(count, sh_scan, &total);
-    sh_start[d] = static_cast<uint32_t>(start);
+#pragma unroll
+    for (int w = 0; w < kSortWarps; ++w) sh_warp[w][d] += static_cast<uint32_t>(start);
     sh_goff[d] = static_cast<int32_t>(static_cast<int64_t>(slot) - start);
     __syncthreads();
-    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_start, sh_keys, sh_vals);
+    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_keys, sh_vals);
     __syncthreads();
     write_tile(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
 }

@@ -206,3 +206,15 @@ def test_roofline_uses_dram_traffic_when_recorded(monkeypatch):
     assert r["l2_gather_gbs"] == round(gathered / 2e-3 / 1e9, 1)
     assert r["frac_l2"] == pytest.approx(gathered / 2e-3 / 1e9 / 20000.0, abs=1e-4)
     assert r["l2_ceiling_row_bytes"] == 512  # fp32 grad_out slices of dim 128
+
+
+def test_roofline_of_a_streaming_kernel_uses_its_algorithmic_bytes(monkeypatch):
+    # the sort can be the longest component (e.g. with serialised launches); it has
+    # no reuse, so its algorithmic bytes are its compulsory ones
+    w = wl.scaled(wl.get_workload("cfg5"), num_tables=2, batch=3, rows=10)
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, off, weighted=False)
+    monkeypatch.setattr(bench, "recorded_traffic", lambda k, wl_: None)
+    r = bench.roofline_of("x", {"bwd.sort": 3.0, "bwd.reduce": 1.0}, {"bwd.sort": 9e9, "bwd.reduce": 1e9},
+                          {"bwd.reduce": 1e8}, 5000.0, "measured", None, [c], w)
+    assert r["kernel"] == "bwd.sort" and r["basis"] == "algorithmic" and r["frac"] == pytest.approx(0.6)
