@@ -546,9 +546,25 @@ def run_l2_ceiling(dev, reps: int = 5):
         ms = statistics.median(a.elapsed_time(b) for a, b in ev)
         res[str(row_bytes)] = {"gbs": round(n * row_bytes / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
                                "rows": n, "set_mb": round(R * row_bytes / 1e6, 1)}
+        # the same rows fetched by TMA gather4
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+        for _ in range(2):
+            tbe.gather_ceiling(rows, idx, out, tma=True, error=err)
+        torch.cuda.synchronize()
+        for a, b in ev:
+            a.record()
+            tbe.gather_ceiling(rows, idx, out, tma=True, error=err)
+            b.record()
+        torch.cuda.synchronize()
+        if int(err.item()) != 0:
+            raise RuntimeError("a bounded wait of the TMA gather probe ran out")
+        ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+        res[str(row_bytes)]["tma_gbs"] = round(n * row_bytes / (ms * 1e-3) / 1e9, 1)
+        res[str(row_bytes)]["tma_ms"] = round(ms, 4)
         del rows, idx, out
     res["how"] = ("cb_gather_ceiling: one warp per 32 random rows of an L2-resident set, 16 bytes per "
-                  "lane, 8 row steps in flight (the walkers' load shape without their bookkeeping)")
+                  "lane, 8 row steps in flight (the walkers' load shape without their bookkeeping); "
+                  "tma_*: cb_gather_ceiling_tma, four rows per TMA gather4, 8 gathers in flight per warp")
     return res
 
 

@@ -227,6 +227,20 @@ cb_status cb_tbe_sorted_payloads(const cb_tbe* h, uint32_t* out, int64_t num_ind
 cb_status cb_gather_ceiling(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* indices,
                             int64_t num_indices, float* out, cudaStream_t stream);
 
+/* The same measurement with the rows fetched by the tensor memory accelerator
+ * (TMA): four rows per cp.async.bulk.tensor .tile::gather4 into shared memory,
+ * eight gathers in flight per warp, completion signalled on an mbarrier. The
+ * rows are read through a 2-D tensor map over `rows` (fp32, num_rows rows of
+ * row_bytes), encoded on the host at every call. Arguments and output as in
+ * cb_gather_ceiling, except:
+ *   num_rows   1 .. 2^31 - 1; a row number >= num_rows reads row 0
+ *   row_bytes  256 or 512
+ *   error      device int, set to CB_ERR_TIMEOUT if a bounded wait on an
+ *              mbarrier ran out (the kernel then stops; out is incomplete)
+ * CB_ERR_CUDA when the driver's tensor-map encoder cannot be reached. */
+cb_status cb_gather_ceiling_tma(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* indices,
+                                int64_t num_indices, float* out, int* error, cudaStream_t stream);
+
 /* Short English description of a status code. */
 const char* cb_tbe_status_string(cb_status s);
 

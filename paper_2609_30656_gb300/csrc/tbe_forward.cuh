@@ -48,6 +48,19 @@ struct FwdPolicy {
     __device__ __forceinline__ Raw fetch(int64_t q) const {
         return {load_index(P.indices, q, P.is32), WEIGHTED ? __ldg(P.weights + q) : 1.f};
     }
+    // The same payload staged in shared memory (index in the first 8 bytes, the
+    // weight after it).
+    static constexpr int kStageBytes = WEIGHTED ? 16 : 8;
+    __device__ __forceinline__ void stage(char* dst, int64_t q) const {
+        if (P.is32) cp_async4(dst, static_cast<const int*>(P.indices) + q);
+        else cp_async8(dst, static_cast<const long long*>(P.indices) + q);
+        if (WEIGHTED) cp_async4(dst + 8, P.weights + q);
+    }
+    __device__ __forceinline__ Raw staged(const char* src) const {
+        const int64_t r = P.is32 ? static_cast<int64_t>(*reinterpret_cast<const int*>(src))
+                                 : static_cast<int64_t>(*reinterpret_cast<const long long*>(src));
+        return {r, WEIGHTED ? *reinterpret_cast<const float*>(src + 8) : 1.f};
+    }
     // Row id of a lookup, checked once here; an out-of-range id contributes nothing.
     __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
         w = x.w;
@@ -116,6 +129,12 @@ struct FwdPolicy {
 #define CB_GATHER_ASYNC 0
 #endif
 constexpr int kGatherAsync = CB_GATHER_ASYNC;
+// Batches of lookup payloads (indices, weights) staged ahead in shared memory
+// by cp.async (0: loaded into registers one batch ahead).
+#ifndef CB_INDEX_STAGE
+#define CB_INDEX_STAGE 0
+#endif
+constexpr int kIndexStage = CB_INDEX_STAGE;
 
 // 16-byte slots per lane of a warp's ring: (groups in flight + 1) load groups.
 template <class Pol, int GC>
@@ -163,6 +182,11 @@ __global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
                 constexpr int kSlots = gather_ring_slots<FwdPolicy<DT, VPL, WEIGHTED>, GC>();
                 walk_rows<FwdPolicy<DT, VPL, WEIGHTED>, GC, kGatherAsync>(
                     pol, c, P.zero_row, lane, slots[threadIdx.x >> 5], ring + (threadIdx.x >> 5) * kSlots * 32);
+            } else if constexpr (kIndexStage > 0) {
+                using Pol = FwdPolicy<DT, VPL, WEIGHTED>;
+                __shared__ __align__(16) char stage[kWarpThreads / 32][(kIndexStage + 1) * 32 * Pol::kStageBytes];
+                walk_rows<Pol, GC, 0, kIndexStage>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5], nullptr,
+                                                  stage[threadIdx.x >> 5]);
             } else {
                 walk_rows<FwdPolicy<DT, VPL, WEIGHTED>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
             }

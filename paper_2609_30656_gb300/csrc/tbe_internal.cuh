@@ -254,12 +254,28 @@ __device__ __forceinline__ void unpack<CB_BF16>(const uint4& r, float (&f)[8]) {
 
 // ---------------------------------------------------------------- output rows
 
+// Cache hints for data touched once per call (CB_STREAM_HINTS): outputs
+// stored with evict-first (st.global.cs), so that they leave L2 before the
+// rows the walkers gather again, and one-pass payload streams loaded with it.
+#ifndef CB_STREAM_HINTS
+#define CB_STREAM_HINTS 1
+#endif
+__device__ __forceinline__ void store_stream(float4* p, float4 v) {
+    if (CB_STREAM_HINTS) __stcs(p, v);
+    else *p = v;
+}
+__device__ __forceinline__ void store_stream(uint2* p, uint2 v) {
+    if (CB_STREAM_HINTS) __stcs(p, v);
+    else *p = v;
+}
+__device__ __forceinline__ uint32_t load_stream(const uint32_t* p) { return CB_STREAM_HINTS ? __ldcs(p) : __ldg(p); }
+
 // Four consecutive columns of an output row, stored as fp32 or rounded to
 // fp16 / bf16 (round to nearest even).
 __device__ __forceinline__ void store_out4(void* row, int64_t col, float a, float b, float c, float d,
                                            int dtype) {
     if (dtype == CB_F32) {
-        *reinterpret_cast<float4*>(static_cast<float*>(row) + col) = make_float4(a, b, c, d);
+        store_stream(reinterpret_cast<float4*>(static_cast<float*>(row) + col), make_float4(a, b, c, d));
         return;
     }
     uint2 w;
@@ -272,7 +288,7 @@ __device__ __forceinline__ void store_out4(void* row, int64_t col, float a, floa
         memcpy(&w.x, &lo, 4);
         memcpy(&w.y, &hi, 4);
     }
-    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(row) + col) = w;
+    store_stream(reinterpret_cast<uint2*>(static_cast<uint16_t*>(row) + col), w);
 }
 
 __host__ __device__ __forceinline__ int dtype_bytes(int dtype) { return dtype == CB_F32 ? 4 : 2; }
@@ -571,6 +587,18 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
                  "l"(gmem)
                  : "memory");
 }
+__device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(
+                     static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(
+                     static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem)
+                 : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() {
@@ -578,9 +606,14 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
 
-template <class Pol, int G, int D = 0>
+// KS > 0 (with D = 0): the items' raw payloads (indices and weights, or
+// sorted payloads) are staged with cp.async KS batches ahead into a per-warp
+// ring of KS + 1 batch slots (Pol::kStageBytes per lane), instead of being
+// loaded into registers one batch ahead.
+template <class Pol, int G, int D = 0, int KS = 0>
 __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uint4* zero_row,
-                                          int lane, EndSlot* slots, uint4* ring = nullptr) {
+                                          int lane, EndSlot* slots, uint4* ring = nullptr,
+                                          char* stage = nullptr) {
     static_assert(G == 1 || G == 2 || G == 4 || G == 8, "rows per warp step");
     static_assert(Pol::kVpl == 1, "one vector per lane");
     constexpr int E = Pol::kElems;
@@ -825,12 +858,33 @@ __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uin
     }
 
     typename Pol::Raw nxt = Pol::none();
-    if (lane < len) nxt = pol.fetch(c.k0 + lane);
+    constexpr int kStage = KS > 0 ? KS : 1;
+    auto stage_slot = [&](int k) { return stage + (k * 32 + lane) * Pol::kStageBytes; };
+    int srd = 0;  // staging slot of the batch read next
+    if constexpr (KS > 0) {
+#pragma unroll
+        for (int k = 0; k < kStage; ++k) {
+            if (k * 32 + lane < len) pol.stage(stage_slot(k), c.k0 + k * 32 + lane);
+            cp_async_commit();
+        }
+    } else {
+        if (lane < len) nxt = pol.fetch(c.k0 + lane);
+    }
     for (int32_t base = 0; base < len; base += 32) {
         const int nb = min(32, len - base);
-        const typename Pol::Raw cur = nxt;
-        nxt = Pol::none();
-        if (base + 32 + lane < len) nxt = pol.fetch(c.k0 + base + 32 + lane);
+        typename Pol::Raw cur = nxt;
+        if constexpr (KS > 0) {
+            cp_async_wait<kStage - 1>();
+            cur = lane < nb ? pol.staged(stage_slot(srd)) : Pol::none();
+            // refill the slot read one batch ago with the batch KS ahead
+            const int swr = srd == 0 ? kStage : srd - 1;
+            if (base + kStage * 32 + lane < len) pol.stage(stage_slot(swr), c.k0 + base + kStage * 32 + lane);
+            cp_async_commit();
+            srd = srd == kStage ? 0 : srd + 1;
+        } else {
+            nxt = Pol::none();
+            if (base + 32 + lane < len) nxt = pol.fetch(c.k0 + base + 32 + lane);
+        }
         uint32_t my_a = kInvalid;
         float my_w = 0.f;
         if (lane < nb) pol.decode(cur, my_a, my_w);
@@ -865,6 +919,10 @@ __device__ __forceinline__ void walk_rows(Pol& pol, const ChunkCtx& c, const uin
                 ain[x] = 0.f;
             }
         }
+    }
+    if constexpr (KS > 0) {
+        cp_async_wait_all();
+        __syncwarp();
     }
     // Empty segments at the chunk end (last chunk of a table), and chunks with
     // no items; then the piece of the segment that runs past the chunk end.

@@ -181,7 +181,12 @@ struct BwdPolicy {
         uint32_t v;
     };
     __device__ __forceinline__ static Raw none() { return {0xffffffffu}; }
-    __device__ __forceinline__ Raw fetch(int64_t q) const { return {__ldg(O.vals_sorted + q)}; }
+    __device__ __forceinline__ Raw fetch(int64_t q) const { return {load_stream(O.vals_sorted + q)}; }
+    static constexpr int kStageBytes = 4;
+    __device__ __forceinline__ void stage(char* dst, int64_t q) const { cp_async4(dst, O.vals_sorted + q); }
+    __device__ __forceinline__ Raw staged(const char* src) const {
+        return {*reinterpret_cast<const uint32_t*>(src)};
+    }
     // Sorted item: the bag whose grad_out row it gathers, and w_i * s_b.
     __device__ __forceinline__ void decode(const Raw& x, uint32_t& a, float& w) const {
         int64_t bag;
@@ -248,7 +253,8 @@ struct BwdPolicy {
                 float4* d4 = reinterpret_cast<float4*>(dst + vec * kElems);
 #pragma unroll
                 for (int x = 0; x < kElems / 4; ++x)
-                    d4[x] = make_float4(tot[k][4 * x], tot[k][4 * x + 1], tot[k][4 * x + 2], tot[k][4 * x + 3]);
+                    store_stream(d4 + x, make_float4(tot[k][4 * x], tot[k][4 * x + 1], tot[k][4 * x + 2],
+                                                     tot[k][4 * x + 3]));
             }
         }
     }
@@ -293,7 +299,13 @@ __global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
         if (lane == 0) Q.tail_owner[j] = -1;
         if constexpr (GC > 0 && VPL == 1 && CB_ROW_WALKER) {
             __shared__ EndSlot slots[kWarpThreads / 32][32];
+#if defined(CB_REDUCE_STAGE) && CB_REDUCE_STAGE > 0
+            __shared__ __align__(16) char stage[kWarpThreads / 32][(CB_REDUCE_STAGE + 1) * 32 * 4];
+            walk_rows<BwdPolicy<GO, VPL, PACKED, APPLY>, GC, 0, CB_REDUCE_STAGE>(
+                pol, c, P.zero_row, lane, slots[threadIdx.x >> 5], nullptr, stage[threadIdx.x >> 5]);
+#else
             walk_rows<BwdPolicy<GO, VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane, slots[threadIdx.x >> 5]);
+#endif
         } else {
             walk_chunk<BwdPolicy<GO, VPL, PACKED, APPLY>, GC>(pol, c, P.zero_row, lane);
         }

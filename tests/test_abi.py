@@ -121,3 +121,13 @@ def test_gather_ceiling_rejects_bad_sizes_on_the_host(lib):
     assert f(p(4096), 0, 512, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # no rows
     assert f(p(4096), 100, 512, None, 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # no indices
     assert f(p(4096), 100, 512, None, 0, None, None) == tbe.CB_OK  # nothing to do
+
+
+def test_tma_gather_ceiling_rejects_bad_sizes_on_the_host(lib):
+    from paper_2609_30656_gb300 import tbe
+    p = ctypes.c_void_p
+    f = lib.cb_gather_ceiling_tma
+    assert f(p(4096), 100, 128, p(8192), 64, p(12288), p(16384), None) == tbe.CB_ERR_INVALID_ARG  # row size
+    assert f(p(4096), 2**31, 512, p(8192), 64, p(12288), p(16384), None) == tbe.CB_ERR_INVALID_ARG  # rows
+    assert f(p(4096), 100, 512, p(8192), 64, p(12288), None, None) == tbe.CB_ERR_INVALID_ARG  # no error word
+    assert f(p(4096), 100, 512, None, 0, None, p(16384), None) == tbe.CB_OK  # nothing to do

@@ -20,3 +20,19 @@ def test_sums_of_gathered_rows(row_bytes):
     pad[:n] = rows.double()[idx].sum(1)
     want = pad.view(-1, 32).sum(1)
     assert torch.equal(got.double(), want)  # integers: exact in any order
+
+
+@pytest.mark.parametrize("row_bytes", [256, 512])
+def test_tma_gather4_sums_of_gathered_rows(row_bytes):
+    from paper_2609_30656_gb300 import tbe
+    g = torch.Generator().manual_seed(row_bytes + 1)
+    rows = torch.randint(-8, 9, (3000, row_bytes // 4), generator=g).to(torch.float32)
+    n = 32 * 301 + 7  # several batches per warp and a ragged last batch
+    idx = torch.randint(0, 3000, (n,), generator=g, dtype=torch.int64)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    got = tbe.gather_ceiling(rows.to(DEV), idx.to(torch.int32).to(DEV), tma=True, error=err).cpu()
+    assert int(err.item()) == 0
+    pad = torch.zeros(32 * ((n + 31) // 32), dtype=torch.float64)
+    pad[:n] = rows.double()[idx].sum(1)
+    want = pad.view(-1, 32).sum(1)
+    assert torch.equal(got.double(), want)
