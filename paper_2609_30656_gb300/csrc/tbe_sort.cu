@@ -78,20 +78,22 @@ __device__ __forceinline__ uint32_t shared_add_if(uint32_t* p, uint32_t v, bool 
 #define CB_RANK_BATCH 2
 #endif
 constexpr int kRankBatch = CB_RANK_BATCH;
-static_assert(kSortItems % kRankBatch == 0, "rank batches divide the items");
-
-__device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int tile_count, uint32_t key_base,
+// NT threads per block rank a tile of kSortTile keys, NI = kSortTile / NT per thread.
+template <int NT>
+__device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortTile / NT], int tile_count, uint32_t key_base,
                                           int shift, uint32_t (*sh_warp)[kRadix + 1],
-                                          uint32_t (&rank2)[kSortItems / 2]) {
+                                          uint32_t (&rank2)[kSortTile / NT / 2]) {
+    constexpr int NI = kSortTile / NT;
+    static_assert(NI % kRankBatch == 0, "rank batches divide the items");
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const uint32_t lt_mask = (1u << lane) - 1u;
 #pragma unroll
-    for (int j0 = 0; j0 < kSortItems; j0 += kRankBatch) {
+    for (int j0 = 0; j0 < NI; j0 += kRankBatch) {
         uint32_t d[kRankBatch], peers[kRankBatch], before[kRankBatch];
 #pragma unroll
         for (int i = 0; i < kRankBatch; ++i) {
             const int j = j0 + i;
-            const int local = wid * (32 * kSortItems) + j * 32 + lane;
+            const int local = wid * (32 * NI) + j * 32 + lane;
             d[i] = local < tile_count ? sort_digit(key[j], key_base, shift) : kRadix;
             peers[i] = __match_any_sync(kFull, d[i]);
         }
@@ -118,13 +120,15 @@ __device__ __forceinline__ void rank_tile(const uint32_t (&key)[kSortItems], int
 #ifndef CB_SORT_KV_PAIRS
 #define CB_SORT_KV_PAIRS 0
 #endif
-__device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], const uint32_t (&val)[kSortItems],
-                                             uint32_t (&rank2)[kSortItems / 2], int tile_count, uint32_t key_base,
+template <int NT>
+__device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortTile / NT], const uint32_t (&val)[kSortTile / NT],
+                                             uint32_t (&rank2)[kSortTile / NT / 2], int tile_count, uint32_t key_base,
                                              int shift, const uint32_t (*sh_warp)[kRadix + 1],
                                              uint32_t* sh_keys, uint32_t* sh_vals) {
+    constexpr int NI = kSortTile / NT;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
-    for (int j = 0; j < kSortItems; ++j) {
+    for (int j = 0; j < NI; ++j) {
         const uint32_t dd = sort_digit(key[j], key_base, shift);
         const uint32_t r = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
         const uint32_t pos = (sh_warp[wid][dd] + r) & 0xffffu;  // < 4096 for real items
@@ -132,8 +136,8 @@ __device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], 
                                 : ((rank2[j >> 1] & 0xffff0000u) | pos);
     }
 #pragma unroll
-    for (int j = 0; j < kSortItems; ++j) {
-        const int local = wid * (32 * kSortItems) + j * 32 + lane;
+    for (int j = 0; j < NI; ++j) {
+        const int local = wid * (32 * NI) + j * 32 + lane;
         if (local < tile_count) {
             const uint32_t pos = (j & 1) ? (rank2[j >> 1] >> 16) : (rank2[j >> 1] & 0xffffu);
             if (CB_SORT_KV_PAIRS) {
@@ -149,18 +153,19 @@ __device__ __forceinline__ void scatter_tile(const uint32_t (&key)[kSortItems], 
 // Consecutive shared slots of one digit go to consecutive global slots
 // (destination = sh_goff[digit] + slot). Half a tile at a time: its shared
 // reads, its destinations, its stores.
+template <int NT>
 __device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, uint32_t key_base,
                                            const int32_t* sh_goff, const uint32_t* sh_keys,
                                            const uint32_t* sh_vals) {
     const int tid = threadIdx.x;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-        constexpr int kHalf = kSortItems / 2;
+        constexpr int kHalf = kSortTile / NT / 2;
         uint32_t key[kHalf], val[kHalf];
         int32_t dst[kHalf];
 #pragma unroll
         for (int j = 0; j < kHalf; ++j) {
-            const int i = tid + (h * kHalf + j) * kSortThreads;
+            const int i = tid + (h * kHalf + j) * NT;
             if (CB_SORT_KV_PAIRS) {
                 const uint2 kv = i < tile_count ? reinterpret_cast<const uint2*>(sh_keys)[i] : make_uint2(0u, 0u);
                 key[j] = kv.x;
@@ -172,10 +177,10 @@ __device__ __forceinline__ void write_tile(const SortPass& S, int tile_count, ui
         }
 #pragma unroll
         for (int j = 0; j < kHalf; ++j)
-            dst[j] = sh_goff[sort_digit(key[j], key_base, S.shift)] + tid + (h * kHalf + j) * kSortThreads;
+            dst[j] = sh_goff[sort_digit(key[j], key_base, S.shift)] + tid + (h * kHalf + j) * NT;
 #pragma unroll
         for (int j = 0; j < kHalf; ++j) {
-            const int i = tid + (h * kHalf + j) * kSortThreads;
+            const int i = tid + (h * kHalf + j) * NT;
             if (i < tile_count && dst[j] >= 0 && dst[j] < S.n) {
                 S.keys_out[dst[j]] = key[j];
                 S.vals_out[dst[j]] = val[j];
@@ -222,7 +227,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
     }
     uint32_t rank2[kSortItems / 2];
-    rank_tile(key, tile_count, key_base, S.shift, sh_warp, rank2);
+    rank_tile<kSortThreads>(key, tile_count, key_base, S.shift, sh_warp, rank2);
     __syncthreads();
 
     // Thread d: per-warp exclusive prefix and the tile's count of digit d.
@@ -298,10 +303,10 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
         static_cast<int64_t>(S.digit_base[static_cast<int64_t>(t) * S.base_stride + d]) + excl - start);
     __syncthreads();
 
-    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_keys, sh_vals);
+    scatter_tile<kSortThreads>(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_keys, sh_vals);
     __syncthreads();
     if (sh_abort) return;
-    write_tile(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
+    write_tile<kSortThreads>(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
 }
 
 // ---------------------------------------------------------------- reduce-then-scan
@@ -398,12 +403,23 @@ __global__ void __launch_bounds__(kRadix) radix_offsets_kernel(const SortPass S)
 }
 
 // (d) The scatter of tile blockIdx.x: the ranking of the single-sweep kernel,
-// with the first output slot of every digit read from (c).
-__global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const SortPass S) {
+// with the first output slot of every digit read from (c). NT threads per tile
+// (NT / 32 warps ranking kSortTile / NT keys per thread); threads 0..255 own one
+// digit each in the prefix step.
+#ifndef CB_SCATTER_THREADS
+#define CB_SCATTER_THREADS 256
+#endif
+constexpr int kScatterThreads = CB_SCATTER_THREADS;
+static_assert(kScatterThreads >= kRadix && kSortTile % kScatterThreads == 0, "scatter block shape");
+
+template <int NT>
+__global__ void __launch_bounds__(NT, NT == 256 ? 3 : 1024 / NT) radix_scatter_kernel(const SortPass S) {
+    constexpr int NI = kSortTile / NT;
+    constexpr int NW = NT / 32;
     extern __shared__ __align__(16) uint32_t sh_dyn[];
     uint32_t* sh_keys = sh_dyn;                            // tile-sorted keys
     uint32_t* sh_vals = sh_dyn + kSortTile;                // tile-sorted payloads
-    __shared__ uint32_t sh_warp[kSortWarps][kRadix + 1];   // per-warp counts, then prefixes
+    __shared__ uint32_t sh_warp[NW][kRadix + 1];           // per-warp counts, then prefixes
                                                            // (slot kRadix: positions past the tile)
     __shared__ int32_t sh_goff[kRadix];                    // global destination - local index
     __shared__ int64_t sh_scan[33];
@@ -411,41 +427,46 @@ __global__ void __launch_bounds__(kSortThreads, 3) radix_scatter_kernel(const So
     const int64_t tile = blockIdx.x;
     if (tile >= *S.num_tiles) return;  // the grid is an upper bound on the tiles
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    for (int i = tid; i < kSortWarps * (kRadix + 1); i += kSortThreads) (&sh_warp[0][0])[i] = 0;
-    const uint32_t slot = S.tile_digits[tile * kRadix + tid];  // digit tid's first output slot
+    for (int i = tid; i < NW * (kRadix + 1); i += NT) (&sh_warp[0][0])[i] = 0;
+    // digit tid's first output slot
+    const uint32_t slot = tid < kRadix ? S.tile_digits[tile * kRadix + tid] : 0u;
     const Chunk tc = S.tiles[tile];
     const int64_t tile_base = tc.k0;
     const int tile_count = static_cast<int>(min64(tc.len & 0x7fffffffu, S.n - tile_base));
     const uint32_t key_base = static_cast<uint32_t>(S.tables[tc.table].key_base);
-    uint32_t key[kSortItems], val[kSortItems];
+    uint32_t key[NI], val[NI];
 #pragma unroll
-    for (int j = 0; j < kSortItems; ++j) {
-        const int local = wid * (32 * kSortItems) + j * 32 + lane;
+    for (int j = 0; j < NI; ++j) {
+        const int local = wid * (32 * NI) + j * 32 + lane;
         const bool valid = local < tile_count;
         key[j] = valid ? __ldg(S.keys_in + tile_base + local) : 0u;
         val[j] = valid ? __ldg(S.vals_in + tile_base + local) : 0u;
     }
     __syncthreads();
-    uint32_t rank2[kSortItems / 2];
-    rank_tile(key, tile_count, key_base, S.shift, sh_warp, rank2);
+    uint32_t rank2[NI / 2];
+    rank_tile<NT>(key, tile_count, key_base, S.shift, sh_warp, rank2);
     __syncthreads();
     const int d = tid;
     uint32_t count = 0;
+    if (d < kRadix) {
 #pragma unroll
-    for (int w = 0; w < kSortWarps; ++w) {
-        const uint32_t c = sh_warp[w][d];
-        sh_warp[w][d] = count;
-        count += c;
+        for (int w = 0; w < NW; ++w) {
+            const uint32_t c = sh_warp[w][d];
+            sh_warp[w][d] = count;
+            count += c;
+        }
     }
     int64_t total;
-    const int64_t start = block_excl_scan(count, sh_scan, &total);
+    const int64_t start = block_excl_scan(count, sh_scan, &total);  // threads past 255 add 0
+    if (d < kRadix) {
 #pragma unroll
-    for (int w = 0; w < kSortWarps; ++w) sh_warp[w][d] += static_cast<uint32_t>(start);
-    sh_goff[d] = static_cast<int32_t>(static_cast<int64_t>(slot) - start);
+        for (int w = 0; w < NW; ++w) sh_warp[w][d] += static_cast<uint32_t>(start);
+        sh_goff[d] = static_cast<int32_t>(static_cast<int64_t>(slot) - start);
+    }
     __syncthreads();
-    scatter_tile(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_keys, sh_vals);
+    scatter_tile<NT>(key, val, rank2, tile_count, key_base, S.shift, sh_warp, sh_keys, sh_vals);
     __syncthreads();
-    write_tile(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
+    write_tile<NT>(S, tile_count, key_base, sh_goff, sh_keys, sh_vals);
 }
 
 // ---------------------------------------------------------------- single sweep
@@ -537,7 +558,13 @@ void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     radix_count_kernel<<<grid, kSortThreads, 0, s>>>(S);
     radix_segsum_kernel<<<parts, kRadix, 0, s>>>(S);
     radix_offsets_kernel<<<parts, kRadix, 0, s>>>(S);
-    radix_scatter_kernel<<<grid, kSortThreads, kSortDynSmem, s>>>(S);
+    static bool configured = false;
+    if (!configured) {  // static + dynamic shared memory may pass the 48 KB default
+        cudaFuncSetAttribute(radix_scatter_kernel<kScatterThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSortDynSmem);
+        configured = true;
+    }
+    radix_scatter_kernel<kScatterThreads><<<grid, kScatterThreads, kSortDynSmem, s>>>(S);
 }
 
 void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
