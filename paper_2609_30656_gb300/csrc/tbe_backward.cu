@@ -507,7 +507,7 @@ namespace cbtbe {
 // step's order, so both give the same sums of squares). Nothing is done when
 // the gradient buffers were too small (the backward then wrote no rows).
 #ifndef CB_APPLY_MIN_BLOCKS
-#define CB_APPLY_MIN_BLOCKS 3  // resident blocks per SM for rows of up to 128 columns (wider: 2)
+#define CB_APPLY_MIN_BLOCKS 4  // resident blocks per SM for rows of up to 128 columns (wider: 2)
 #endif
 #ifndef CB_APPLY_ROWS_M1
 #define CB_APPLY_ROWS_M1 2  // rows stepped at once for rows of up to 128 columns

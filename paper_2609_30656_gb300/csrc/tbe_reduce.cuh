@@ -87,9 +87,14 @@ __device__ __forceinline__ void step_cols(const TableDev& td, int64_t row, int c
     store_step(p, td.dtype, col, load_cols(p, td.dtype, col), g, scale);
 }
 
-// This lane's share of sum g^2 over four columns (the same expression in the
-// fused and the two-pass step, so both give the same Adagrad state).
-__device__ __forceinline__ float sq4(float4 g) { return g.x * g.x + g.y * g.y + g.z * g.z + g.w * g.w; }
+// This lane's share of sum g^2 over four columns, in one fixed order of
+// roundings (an explicit product and three fused multiply-adds): written as a
+// plain sum of products, the compiler may fuse either product of a pair, and
+// may choose differently in the fused and the two-pass step, which must give
+// the same Adagrad state bit for bit.
+__device__ __forceinline__ float sq4(float4 g) {
+    return fmaf(g.w, g.w, fmaf(g.z, g.z, fmaf(g.y, g.y, __fmul_rn(g.x, g.x))));
+}
 
 // The Adagrad scale from the summed squares and the row's previous state `m0`
 // (meaningful in lane 0); lane 0 stores the new state.
