@@ -78,10 +78,40 @@ __device__ __forceinline__ void find_bag32(const Problem& P, BagWindow32& W, int
     }
 }
 
+// The bags of 32 consecutive positions p0 .. p0 + 31 without shuffles when
+// possible: the window's ends inside the step become bits of a mask (one warp
+// OR), and lane l's bag is the window's first bag plus the ends at or before
+// p0 + l. Returns false (nothing written) when two ends coincide (an empty bag)
+// or the step reaches past the window's last end; the caller then bisects.
+#ifndef CB_KEYGEN_MASK
+#define CB_KEYGEN_MASK 1
+#endif
+__device__ __forceinline__ bool bags_by_mask(const BagWindow32& W, int32_t p0, int lane, bool want_range,
+                                             int64_t& bag, int32_t& s, int32_t& e) {
+    const bool before = W.my_end < p0;
+    const bool inside = W.my_end >= p0 && W.my_end <= p0 + 31;
+    const uint32_t nbefore = __popc(__ballot_sync(kFull, before));
+    const uint32_t nin = __popc(__ballot_sync(kFull, inside));
+    const uint32_t mask = __reduce_or_sync(kFull, inside ? 1u << (W.my_end - p0) : 0u);
+    if (__popc(mask) != static_cast<int>(nin) || nbefore + nin >= 32) return false;  // warp-uniform
+    const uint32_t le = lane == 31 ? kFull : (2u << lane) - 1u;
+    const int cnt = static_cast<int>(nbefore) + __popc(mask & le);
+    bag = W.win + cnt;
+    if (want_range) {
+        e = __shfl_sync(kFull, W.my_end, cnt);
+        const int32_t prev = __shfl_sync(kFull, W.my_end, cnt > 0 ? cnt - 1 : 0);
+        s = cnt > 0 ? prev : W.win_start;
+    }
+    return true;
+}
+
 // A warp walks one chunk kKeygenSteps x 32 lookups at a time: the indices (and
 // weights) of all the steps are loaded first, so that many loads are in flight
 // per warp, then each step finds its lanes' bags and writes.
-constexpr int kKeygenSteps = 8;
+#ifndef CB_KEYGEN_STEPS
+#define CB_KEYGEN_STEPS 12
+#endif
+constexpr int kKeygenSteps = CB_KEYGEN_STEPS;
 
 template <bool PACKED>
 __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q, KeyGen K) {
@@ -115,8 +145,9 @@ __global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q,
                 if (base + 32 * u >= len) break;  // warp-uniform
                 const bool valid = q < len;
                 int64_t my_bag;
-                int32_t my_s, my_e;
-                find_bag32(P, W, bag_hi, k0, q, valid, lane, my_bag, my_s, my_e);
+                int32_t my_s = 0, my_e = 0;
+                if (!CB_KEYGEN_MASK || !bags_by_mask(W, base + 32 * u, lane, PACKED && P.mean, my_bag, my_s, my_e))
+                    find_bag32(P, W, bag_hi, k0, q, valid, lane, my_bag, my_s, my_e);
                 if (!valid) continue;
                 if (my_bag >= bag_hi) {  // only reachable with malformed offsets
                     set_error(P.error, CB_ERR_BAD_OFFSETS);
