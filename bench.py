@@ -365,6 +365,8 @@ def run_ours(args):
     ceiling = None if args.no_l2 else run_l2_ceiling(dev)
     roofline = roofline_of(w.name, comp_ms, comp_bytes, comp_compulsory, peak, peak_kind, ceiling,
                            counts, w)
+    if ceiling and "fwd.gather" in components:
+        components["fwd.gather"].update(gather_vs_l2(comp_ms["fwd.gather"], counts, w, ceiling))
     mean_counts_n = statistics.mean(c.n for c in counts)
     fwd_bytes_step = fwd_b / args.steps
     bwd_bytes_step = bwd_b / args.steps
@@ -520,6 +522,22 @@ def roofline_of(workload, comp_ms, comp_bytes, comp_compulsory, peak, peak_kind,
     return r
 
 
+def gather_vs_l2(ms: float, counts, w, ceiling) -> dict:
+    """The forward gather's row bytes per second against the L2 random-gather
+    rate of rows of its size: plain fp32 sums (`frac_l2`) and, for half-precision
+    tables, fp16 rows widened into fp32 sums as the gather does (`frac_l2_widened`)."""
+    rows = sum(metrics.forward_bytes(c)["rows"] for c in counts) / len(counts)
+    key = str(min(512, w.elem_bytes * max(w.dims)))
+    if key not in ceiling:
+        return {}
+    gbs = rows / (ms * 1e-3) / 1e9
+    r = {"l2_gather_gbs": round(gbs, 1), "frac_l2": round(gbs / ceiling[key]["gbs"], 4),
+         "l2_ceiling_row_bytes": int(key)}
+    if w.dtype == "f16" and "f16_sum_gbs" in ceiling[key]:
+        r["frac_l2_widened"] = round(gbs / ceiling[key]["f16_sum_gbs"], 4)
+    return r
+
+
 def run_l2_ceiling(dev, reps: int = 5):
     """cb_gather_ceiling on a 33.5 MB row set (one cfg5 table's grad_out slice,
     [65536, 128] fp32) for 512- and 256-byte rows: 2^25 uniformly random rows
@@ -561,10 +579,25 @@ def run_l2_ceiling(dev, reps: int = 5):
         ms = statistics.median(a.elapsed_time(b) for a, b in ev)
         res[str(row_bytes)]["tma_gbs"] = round(n * row_bytes / (ms * 1e-3) / 1e9, 1)
         res[str(row_bytes)]["tma_ms"] = round(ms, 4)
-        del rows, idx, out
+        # fp16 rows of the same size, widened into fp32 sums as the forward does
+        rows16 = torch.randn(R, row_bytes // 2, generator=g, device=dev).to(torch.float16)
+        for _ in range(2):
+            tbe.gather_ceiling(rows16, idx, out)
+        torch.cuda.synchronize()
+        for a, b in ev:
+            a.record()
+            tbe.gather_ceiling(rows16, idx, out)
+            b.record()
+        torch.cuda.synchronize()
+        ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+        res[str(row_bytes)]["f16_sum_gbs"] = round(n * row_bytes / (ms * 1e-3) / 1e9, 1)
+        res[str(row_bytes)]["f16_sum_ms"] = round(ms, 4)
+        del rows, rows16, idx, out
     res["how"] = ("cb_gather_ceiling: one warp per 32 random rows of an L2-resident set, 16 bytes per "
                   "lane, 8 row steps in flight (the walkers' load shape without their bookkeeping); "
-                  "tma_*: cb_gather_ceiling_tma, four rows per TMA gather4, 8 gathers in flight per warp")
+                  "tma_*: cb_gather_ceiling_tma, four rows per TMA gather4, 8 gathers in flight per warp; "
+                  "f16_sum_*: cb_gather_ceiling_f16, fp16 rows of the same size widened into fp32 sums "
+                  "(the forward's 8 mixed-precision adds per 16 bytes)")
     return res
 
 

@@ -227,6 +227,16 @@ cb_status cb_tbe_sorted_payloads(const cb_tbe* h, uint32_t* out, int64_t num_ind
 cb_status cb_gather_ceiling(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* indices,
                             int64_t num_indices, float* out, cudaStream_t stream);
 
+/* The same measurement on half-precision rows with the forward's arithmetic:
+ * `rows` read as fp16 and every value widened into fp32 sums by the
+ * mixed-precision add (8 adds per 16 bytes, the forward gather's work per
+ * stored value on fp16 tables). The rate it reaches bounds the forward gather
+ * on half-precision tables served from L2. Arguments, output and errors as in
+ * cb_gather_ceiling (out[k]: the fp32 sum of every fp16 value of the rows of
+ * items 32k .. 32k + 31). */
+cb_status cb_gather_ceiling_f16(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* indices,
+                                int64_t num_indices, float* out, cudaStream_t stream);
+
 /* The same measurement with the rows fetched by the tensor memory accelerator
  * (TMA): four rows per cp.async.bulk.tensor .tile::gather4 into shared memory,
  * eight gathers in flight per warp, completion signalled on an mbarrier. The

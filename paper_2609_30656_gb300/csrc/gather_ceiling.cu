@@ -25,7 +25,10 @@ namespace {
 
 constexpr int kRows = 8;  // row steps in flight per lane (the fp32 reduce's setting)
 
-template <int G>
+// DT: CB_F32 rows summed with fp32 adds (the reduce's grad_out slices), or
+// CB_F16 rows widened into fp32 sums by the mixed-precision add, the
+// forward's arithmetic on half-precision tables (8 adds per 16 bytes).
+template <int G, int DT>
 __global__ void __launch_bounds__(kWarpThreads) gather_ceiling_kernel(const uint4* __restrict__ rows,
                                                                       uint32_t stride, int64_t num_rows,
                                                                       const uint32_t* __restrict__ idx,
@@ -41,7 +44,10 @@ __global__ void __launch_bounds__(kWarpThreads) gather_ceiling_kernel(const uint
         uint32_t my = q < n ? __ldg(idx + q) : 0u;
         if (my >= num_rows) my = 0;  // kept inside the row set whatever the indices hold
         const bool live = q < n;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        constexpr int E = DT == CB_F32 ? 4 : 8;
+        float acc[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = 0.f;
 #pragma unroll
         for (int s0 = 0; s0 < kSteps; s0 += UG) {
             uint4 x[UG];
@@ -56,20 +62,19 @@ __global__ void __launch_bounds__(kWarpThreads) gather_ceiling_kernel(const uint
 #pragma unroll
             for (int u = 0; u < UG; ++u) {
                 if (!ok[u]) continue;
-                acc[0] += __uint_as_float(x[u].x);
-                acc[1] += __uint_as_float(x[u].y);
-                acc[2] += __uint_as_float(x[u].z);
-                acc[3] += __uint_as_float(x[u].w);
+                accumulate<DT, false>(acc, x[u], 1.f);
             }
         }
-        float t = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+        float t = 0.f;
+#pragma unroll
+        for (int e = 0; e < E; ++e) t += acc[e];
 #pragma unroll
         for (int off = 16; off >= 1; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
         if (lane == 0) out[b] = t;
     }
 }
 
-template <int G>
+template <int G, int DT>
 cb_status launch(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* idx, int64_t n,
                  float* out, cudaStream_t s) {
     int dev = 0, sms = 1;
@@ -78,10 +83,10 @@ cb_status launch(const void* rows, int64_t num_rows, int32_t row_bytes, const ui
         cudaGetLastError();
         return CB_ERR_CUDA;
     }
-    const int cap = occupancy_grid(gather_ceiling_kernel<G>, kWarpThreads, sms);
+    const int cap = occupancy_grid(gather_ceiling_kernel<G, DT>, kWarpThreads, sms);
     const int64_t need = ((n + 31) / 32 + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
     const int grid = static_cast<int>(need < cap ? (need > 0 ? need : 1) : cap);
-    gather_ceiling_kernel<G><<<grid, kWarpThreads, 0, s>>>(static_cast<const uint4*>(rows),
+    gather_ceiling_kernel<G, DT><<<grid, kWarpThreads, 0, s>>>(static_cast<const uint4*>(rows),
                                                             static_cast<uint32_t>(row_bytes / 16), num_rows,
                                                             idx, n, out);
     return cudaGetLastError() == cudaSuccess ? CB_OK : CB_ERR_CUDA;
@@ -90,21 +95,38 @@ cb_status launch(const void* rows, int64_t num_rows, int32_t row_bytes, const ui
 }  // namespace
 }  // namespace cbtbe
 
-extern "C" cb_status cb_gather_ceiling(const void* rows, int64_t num_rows, int32_t row_bytes,
-                                       const uint32_t* indices, int64_t num_indices, float* out,
-                                       cudaStream_t stream) {
-    using namespace cbtbe;
+namespace cbtbe {
+namespace {
+
+template <int DT>
+cb_status gather_ceiling(const void* rows, int64_t num_rows, int32_t row_bytes, const uint32_t* indices,
+                         int64_t num_indices, float* out, cudaStream_t stream) {
     if (!rows || num_rows <= 0 || num_rows > (int64_t(1) << 32) || num_indices < 0 ||
         (num_indices > 0 && (!indices || !out)) || (reinterpret_cast<uintptr_t>(rows) & 15u))
         return CB_ERR_INVALID_ARG;
     if (num_indices == 0) return CB_OK;
     switch (row_bytes) {
-        case 512: return launch<1>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
-        case 256: return launch<2>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
-        case 128: return launch<4>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
-        case 64: return launch<8>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
+        case 512: return launch<1, DT>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
+        case 256: return launch<2, DT>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
+        case 128: return launch<4, DT>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
+        case 64: return launch<8, DT>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
         default: return CB_ERR_INVALID_ARG;
     }
+}
+
+}  // namespace
+}  // namespace cbtbe
+
+extern "C" cb_status cb_gather_ceiling(const void* rows, int64_t num_rows, int32_t row_bytes,
+                                       const uint32_t* indices, int64_t num_indices, float* out,
+                                       cudaStream_t stream) {
+    return cbtbe::gather_ceiling<CB_F32>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
+}
+
+extern "C" cb_status cb_gather_ceiling_f16(const void* rows, int64_t num_rows, int32_t row_bytes,
+                                           const uint32_t* indices, int64_t num_indices, float* out,
+                                           cudaStream_t stream) {
+    return cbtbe::gather_ceiling<CB_F16>(rows, num_rows, row_bytes, indices, num_indices, out, stream);
 }
 
 // ---------------------------------------------------------------- TMA gather4

@@ -33,7 +33,7 @@ EXPORTS = ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward
            "cb_tbe_launch_count", "cb_tbe_status_string", "cb_tbe_destroy",
            "cb_tbe_forward_noalloc", "cb_fm_forward", "cb_fm_backward", "cb_tbe_weight_grad",
            "cb_tbe_backward_apply", "cb_tbe_apply_sparse", "cb_kjt_replicate",
-           "cb_tbe_sorted_payloads", "cb_gather_ceiling", "cb_gather_ceiling_tma")
+           "cb_tbe_sorted_payloads", "cb_gather_ceiling", "cb_gather_ceiling_f16", "cb_gather_ceiling_tma")
 
 
 class CbTableDesc(ctypes.Structure):
@@ -90,13 +90,14 @@ def load_library() -> ctypes.CDLL:
     lib.cb_kjt_replicate.argtypes = [p, p, p, ctypes.c_int, i32, i32, i64, i32, p, p, p, p]
     lib.cb_tbe_sorted_payloads.argtypes = [p, p, i64, p]
     lib.cb_gather_ceiling.argtypes = [p, i64, i32, p, i64, p, p]
+    lib.cb_gather_ceiling_f16.argtypes = [p, i64, i32, p, i64, p, p]
     lib.cb_gather_ceiling_tma.argtypes = [p, i64, i32, p, i64, p, p, p]
     lib.cb_fm_forward.argtypes = [p, i32, i32, i32, i64, p, p]
     lib.cb_fm_backward.argtypes = [p, p, i32, i32, i32, i64, p, p]
     for name in ("cb_tbe_create", "cb_tbe_reserve", "cb_tbe_forward", "cb_tbe_backward",
                  "cb_tbe_get_error", "cb_tbe_last_timings", "cb_fm_forward", "cb_fm_backward",
                  "cb_tbe_weight_grad", "cb_tbe_backward_apply", "cb_kjt_replicate",
-                 "cb_tbe_sorted_payloads", "cb_gather_ceiling", "cb_gather_ceiling_tma"):
+                 "cb_tbe_sorted_payloads", "cb_gather_ceiling", "cb_gather_ceiling_f16", "cb_gather_ceiling_tma"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -422,10 +423,13 @@ def gather_ceiling(rows: torch.Tensor, indices: torch.Tensor, out: torch.Tensor 
     """Random-row gather out of `rows` ([R, row_bytes / 4] fp32, L2-sized) at `indices`
     (int32 viewed as uint32) with the walkers' load shape (cb_gather_ceiling), or by TMA
     gather4 (tma=True, cb_gather_ceiling_tma; `error` an int32 [1] device word); returns
-    the per-32-item sums."""
+    the per-32-item sums. With fp16 rows ([R, row_bytes / 2]) the values are widened
+    into fp32 sums as the forward does (cb_gather_ceiling_f16)."""
     lib = load_library()
-    if rows.device.type != "cuda" or rows.dtype != torch.float32 or rows.dim() != 2 or not rows.is_contiguous():
-        raise ValueError("rows must be a contiguous 2-D fp32 CUDA tensor")
+    half = rows.dtype == torch.float16
+    if (rows.device.type != "cuda" or rows.dtype not in (torch.float32, torch.float16) or rows.dim() != 2
+            or not rows.is_contiguous() or (half and tma)):
+        raise ValueError("rows must be a contiguous 2-D fp32 (or, without tma, fp16) CUDA tensor")
     if indices.device != rows.device or indices.dtype != torch.int32:
         raise ValueError("indices must be int32 on the device of rows")
     n = indices.numel()
@@ -439,6 +443,10 @@ def gather_ceiling(rows: torch.Tensor, indices: torch.Tensor, out: torch.Tensor 
             _check(lib.cb_gather_ceiling_tma(_ptr(rows), rows.shape[0], rows.shape[1] * 4,
                                              _ptr(indices.contiguous()), n, _ptr(out), _ptr(error), stream),
                    "cb_gather_ceiling_tma")
+        elif half:
+            _check(lib.cb_gather_ceiling_f16(_ptr(rows), rows.shape[0], rows.shape[1] * 2,
+                                             _ptr(indices.contiguous()), n, _ptr(out), stream),
+                   "cb_gather_ceiling_f16")
         else:
             _check(lib.cb_gather_ceiling(_ptr(rows), rows.shape[0], rows.shape[1] * 4, _ptr(indices.contiguous()),
                                          n, _ptr(out), stream), "cb_gather_ceiling")

@@ -112,10 +112,11 @@ def test_create_refuses_a_key_space_beyond_32_bits(lib):
     assert lib.cb_tbe_create(descs, 2, 0, 1, 0, ctypes.byref(h)) == tbe.CB_ERR_INVALID_ARG
 
 
-def test_gather_ceiling_rejects_bad_sizes_on_the_host(lib):
+@pytest.mark.parametrize("name", ["cb_gather_ceiling", "cb_gather_ceiling_f16"])
+def test_gather_ceiling_rejects_bad_sizes_on_the_host(lib, name):
     from paper_2609_30656_gb300 import tbe
     p = ctypes.c_void_p
-    f = lib.cb_gather_ceiling
+    f = getattr(lib, name)
     assert f(p(4096), 100, 96, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # row size
     assert f(p(4100), 100, 512, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # alignment
     assert f(p(4096), 0, 512, p(8192), 64, p(12288), None) == tbe.CB_ERR_INVALID_ARG  # no rows

@@ -208,6 +208,22 @@ def test_roofline_uses_dram_traffic_when_recorded(monkeypatch):
     assert r["l2_ceiling_row_bytes"] == 512  # fp32 grad_out slices of dim 128
 
 
+def test_forward_gather_against_both_l2_rates():
+    # fp16 rows of dim 128 (256 bytes): against the plain gather rate and the
+    # rate with the forward's widening adds
+    w = wl.scaled(wl.get_workload("cfg5"), num_tables=2, batch=3, rows=10)
+    off = torch.tensor([0, 2, 2, 5, 6, 7, 7])
+    c = metrics.batch_counts(w.dims, w.elem_bytes, w.batch, off, weighted=False)
+    rows = 7 * 128 * 2  # 7 lookups of 256-byte rows
+    assert metrics.forward_bytes(c)["rows"] == rows
+    ceiling = {"256": {"gbs": 20000.0, "f16_sum_gbs": 16000.0}}
+    r = bench.gather_vs_l2(1e-6, [c], w, ceiling)  # 1 ns
+    assert r["l2_gather_gbs"] == round(rows / 1e-9 / 1e9, 1) and r["l2_ceiling_row_bytes"] == 256
+    assert r["frac_l2"] == pytest.approx(rows / 1e-9 / 1e9 / 20000.0, abs=1e-4)
+    assert r["frac_l2_widened"] == pytest.approx(rows / 1e-9 / 1e9 / 16000.0, abs=1e-4)
+    assert bench.gather_vs_l2(1e-6, [c], w, {"512": {"gbs": 1.0}}) == {}
+
+
 def test_roofline_of_a_streaming_kernel_uses_its_algorithmic_bytes(monkeypatch):
     # the sort can be the longest component (e.g. with serialised launches); it has
     # no reuse, so its algorithmic bytes are its compulsory ones

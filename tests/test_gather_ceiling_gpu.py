@@ -36,3 +36,17 @@ def test_tma_gather4_sums_of_gathered_rows(row_bytes):
     pad[:n] = rows.double()[idx].sum(1)
     want = pad.view(-1, 32).sum(1)
     assert torch.equal(got.double(), want)
+
+
+@pytest.mark.parametrize("row_bytes", [128, 256, 512])
+def test_half_rows_widened_into_fp32_sums(row_bytes):
+    from paper_2609_30656_gb300 import tbe
+    g = torch.Generator().manual_seed(row_bytes + 2)
+    rows = torch.randint(-8, 9, (1500, row_bytes // 2), generator=g).to(torch.float16)
+    n = 32 * 123 + 9  # a ragged last batch
+    idx = torch.randint(0, 1500, (n,), generator=g, dtype=torch.int64)
+    got = tbe.gather_ceiling(rows.to(DEV), idx.to(torch.int32).to(DEV)).cpu()
+    pad = torch.zeros(32 * ((n + 31) // 32), dtype=torch.float64)
+    pad[:n] = rows.double()[idx].sum(1)
+    want = pad.view(-1, 32).sum(1)
+    assert torch.equal(got.double(), want)  # integers: exact in any order
