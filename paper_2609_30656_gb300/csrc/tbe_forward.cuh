@@ -26,6 +26,7 @@ struct FwdPolicy {
     static constexpr bool kTwoLevel = DT == CB_F32;  // half rows: one fp32 level (registers)
     static constexpr bool kUnrollGroups = CB_WALK_UNROLL_GROUPS;
     static constexpr bool kFastBatch = CB_WALK_FAST_BATCH;
+    static constexpr int kPrefetch = CB_WALK_PREFETCH;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;

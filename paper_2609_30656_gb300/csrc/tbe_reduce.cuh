@@ -165,6 +165,7 @@ struct BwdPolicy {
     static constexpr bool kWeighted = PACKED;
     static constexpr bool kUnrollGroups = GO == CB_F32 ? CB_REDUCE_UNROLL_GROUPS : false;
     static constexpr bool kFastBatch = GO == CB_F32 ? CB_REDUCE_FAST_BATCH : CB_REDUCE_HALF_FAST_BATCH;
+    static constexpr int kPrefetch = CB_REDUCE_PREFETCH;
 
     const Problem& P;  // kernel parameters: read in place, not held in registers
     const Plan& Q;
