@@ -23,55 +23,95 @@
 namespace cbtbe {
 namespace {
 
-constexpr int kRows = 8;  // row steps in flight per lane (the fp32 reduce's setting)
+// Row steps in flight per lane, and resident blocks per SM the kernel is
+// compiled for: the rate out of L2 grows with the warps resident per SM more
+// than with the loads each warp has in flight (measured: 4 steps at 8 blocks of
+// 256 threads reach ~21 TB/s for 256-byte rows, fp32 or widened fp16, where 8
+// steps at 4-5 blocks, the register budget of the walkers, reach 15.8-20 TB/s).
+constexpr int kRows = 4;
+
+// x's values added into acc: fp32 adds, or fp16 values widened into the fp32
+// sums by the mixed-precision add (as the forward gather adds them).
+template <int DT>
+__device__ __forceinline__ void add_row(float (&acc)[DT == CB_F32 ? 4 : 8], const uint4& x) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        if constexpr (DT == CB_F32) {
+            acc[i] += __uint_as_float(w[i]);
+        } else {
+            asm("{ .reg .b16 lo, hi;\n\t mov.b32 {lo, hi}, %2;\n\t"
+                " add.rn.f32.f16 %0, lo, %0;\n\t add.rn.f32.f16 %1, hi, %1; }"
+                : "+f"(acc[2 * i]), "+f"(acc[2 * i + 1]) : "r"(w[i]));
+        }
+    }
+}
+
+// The sum of every value of the rows of one batch of 32 items, per lane
+// (lane-summed by the caller). TAIL: the last, partial batch, whose missing
+// items add nothing.
+template <int G, int DT, bool TAIL>
+__device__ __forceinline__ float batch_sum(const uint4* __restrict__ rows, uint32_t my, bool live, int lane) {
+    constexpr int V = 32 / G;            // lanes per row
+    constexpr int kSteps = 32 / G;       // row steps per batch of 32 items
+    constexpr int UG = kRows < kSteps ? kRows : kSteps;
+    constexpr int E = DT == CB_F32 ? 4 : 8;
+    const int g = lane / V, v = lane - g * V;
+    float acc[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] = 0.f;
+#pragma unroll
+    for (int s0 = 0; s0 < kSteps; s0 += UG) {
+        uint4 x[UG];
+        bool ok[UG];
+#pragma unroll
+        for (int u = 0; u < UG; ++u) {
+            const int src = (s0 + u) * G + g;
+            const uint32_t r = __shfl_sync(kFull, my, src);
+            ok[u] = TAIL ? __shfl_sync(kFull, live, src) : true;
+            x[u] = __ldg(rows + static_cast<uint64_t>(r) * V + v);  // a row is V vectors
+        }
+#pragma unroll
+        for (int u = 0; u < UG; ++u)
+            if (!TAIL || ok[u]) add_row<DT>(acc, x[u]);
+    }
+    float t = 0.f;
+#pragma unroll
+    for (int e = 0; e < E; ++e) t += acc[e];
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
+    return t;
+}
 
 // DT: CB_F32 rows summed with fp32 adds (the reduce's grad_out slices), or
 // CB_F16 rows widened into fp32 sums by the mixed-precision add, the
 // forward's arithmetic on half-precision tables (8 adds per 16 bytes).
+// Full batches only; the partial last batch goes to gather_tail_kernel.
 template <int G, int DT>
-__global__ void __launch_bounds__(kWarpThreads) gather_ceiling_kernel(const uint4* __restrict__ rows,
-                                                                      uint32_t stride, int64_t num_rows,
+__global__ void __launch_bounds__(kWarpThreads, 8) gather_ceiling_kernel(const uint4* __restrict__ rows,
+                                                                      int64_t num_rows,
                                                                       const uint32_t* __restrict__ idx,
-                                                                      int64_t n, float* __restrict__ out) {
-    constexpr int V = 32 / G;            // lanes per row
-    constexpr int kSteps = 32 / G;       // row steps per batch of 32 items
-    constexpr int UG = kRows < kSteps ? kRows : kSteps;
+                                                                      int64_t batches, float* __restrict__ out) {
     const int lane = threadIdx.x & 31;
-    const int g = lane / V, v = lane - g * V;
-    const int64_t batches = (n + 31) / 32;
-    for (int64_t b = warp_id_global(); b < batches; b += warps_in_grid()) {
-        const int64_t q = b * 32 + lane;
-        uint32_t my = q < n ? __ldg(idx + q) : 0u;
+    const int64_t warps = static_cast<int64_t>(gridDim.x) * (kWarpThreads / 32);
+    for (int64_t b = (static_cast<int64_t>(blockIdx.x) * kWarpThreads + threadIdx.x) / 32; b < batches; b += warps) {
+        uint32_t my = __ldg(idx + b * 32 + lane);
         if (my >= num_rows) my = 0;  // kept inside the row set whatever the indices hold
-        const bool live = q < n;
-        constexpr int E = DT == CB_F32 ? 4 : 8;
-        float acc[E];
-#pragma unroll
-        for (int e = 0; e < E; ++e) acc[e] = 0.f;
-#pragma unroll
-        for (int s0 = 0; s0 < kSteps; s0 += UG) {
-            uint4 x[UG];
-            bool ok[UG];
-#pragma unroll
-            for (int u = 0; u < UG; ++u) {
-                const int src = (s0 + u) * G + g;
-                const uint32_t r = __shfl_sync(kFull, my, src);
-                ok[u] = __shfl_sync(kFull, live, src);
-                x[u] = __ldg(rows + static_cast<uint64_t>(r) * stride + v);
-            }
-#pragma unroll
-            for (int u = 0; u < UG; ++u) {
-                if (!ok[u]) continue;
-                accumulate<DT, false>(acc, x[u], 1.f);
-            }
-        }
-        float t = 0.f;
-#pragma unroll
-        for (int e = 0; e < E; ++e) t += acc[e];
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
+        const float t = batch_sum<G, DT, false>(rows, my, true, lane);
         if (lane == 0) out[b] = t;
     }
+}
+
+template <int G, int DT>
+__global__ void __launch_bounds__(32) gather_tail_kernel(const uint4* __restrict__ rows, int64_t num_rows,
+                                                         const uint32_t* __restrict__ idx, int64_t b, int64_t n,
+                                                         float* __restrict__ out) {
+    const int lane = threadIdx.x;
+    const int64_t q = b * 32 + lane;
+    uint32_t my = q < n ? __ldg(idx + q) : 0u;
+    if (my >= num_rows) my = 0;
+    const float t = batch_sum<G, DT, true>(rows, my, q < n, lane);
+    if (lane == 0) out[b] = t;
 }
 
 template <int G, int DT>
@@ -83,12 +123,16 @@ cb_status launch(const void* rows, int64_t num_rows, int32_t row_bytes, const ui
         cudaGetLastError();
         return CB_ERR_CUDA;
     }
-    const int cap = occupancy_grid(gather_ceiling_kernel<G, DT>, kWarpThreads, sms);
-    const int64_t need = ((n + 31) / 32 + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
-    const int grid = static_cast<int>(need < cap ? (need > 0 ? need : 1) : cap);
-    gather_ceiling_kernel<G, DT><<<grid, kWarpThreads, 0, s>>>(static_cast<const uint4*>(rows),
-                                                            static_cast<uint32_t>(row_bytes / 16), num_rows,
-                                                            idx, n, out);
+    // rows of row_bytes = (32 / G) * 16: full batches, then the partial last one
+    const uint4* r = static_cast<const uint4*>(rows);
+    const int64_t full = n / 32;
+    if (full > 0) {
+        const int cap = occupancy_grid(gather_ceiling_kernel<G, DT>, kWarpThreads, sms);
+        const int64_t need = (full + (kWarpThreads / 32) - 1) / (kWarpThreads / 32);
+        const int grid = static_cast<int>(need < cap ? need : cap);
+        gather_ceiling_kernel<G, DT><<<grid, kWarpThreads, 0, s>>>(r, num_rows, idx, full, out);
+    }
+    if (n % 32) gather_tail_kernel<G, DT><<<1, 32, 0, s>>>(r, num_rows, idx, full, n, out);
     return cudaGetLastError() == cudaSuccess ? CB_OK : CB_ERR_CUDA;
 }
 

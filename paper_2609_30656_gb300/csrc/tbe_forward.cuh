@@ -147,8 +147,25 @@ __host__ __device__ constexpr int gather_ring_slots() {
     return kGatherAsync > 0 ? (depth + 1) * ug : 0;
 }
 
+// Resident blocks per SM the gather is compiled for. The row walker with one
+// vector per lane and no weights fits 5 blocks' registers (48) without
+// spilling, and the gather's rate out of L2 grows with the warps resident
+// (cfg5: 4.07 -> 3.72 ms from 4 to 5 blocks); the other layouts spill at 48
+// registers and keep 4.
+#ifndef CB_WALK_MIN_BLOCKS_ROW
+#define CB_WALK_MIN_BLOCKS_ROW 5
+#endif
+#ifndef CB_WALK_ROW_WEIGHTED
+#define CB_WALK_ROW_WEIGHTED 0  // 1: weighted row layouts take CB_WALK_MIN_BLOCKS_ROW too
+#endif
+template <int VPL, bool WEIGHTED, int GC>
+constexpr int gather_min_blocks() {
+    return VPL == 1 && GC > 0 && GC != 4 && (!WEIGHTED || CB_WALK_ROW_WEIGHTED) ? CB_WALK_MIN_BLOCKS_ROW
+                                                                                : CB_WALK_MIN_BLOCKS;
+}
+
 template <int DT, int VPL, bool WEIGHTED, int GC>
-__global__ void __launch_bounds__(kWarpThreads, CB_WALK_MIN_BLOCKS)
+__global__ void __launch_bounds__(kWarpThreads, gather_min_blocks<VPL, WEIGHTED, GC>())
     fwd_gather_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q, void* out,
                       int cls) {
     const int lane = threadIdx.x & 31;
