@@ -266,8 +266,22 @@ struct BwdPolicy {
     }
 };
 
+// Resident blocks per SM the reduce is compiled for: half-precision grad_out
+// slices with one vector per lane, no coefficient and no optimizer step fit 5
+// blocks' registers (48) without spilling, and more resident warps raise the
+// rate of the L2-served gathers; fp32 slices (8 rows in flight per lane) and
+// the other forms keep CB_REDUCE_MIN_BLOCKS.
+#ifndef CB_REDUCE_HALF_MIN_BLOCKS
+#define CB_REDUCE_HALF_MIN_BLOCKS 5
+#endif
 template <int GO, int VPL, bool PACKED, int GC, bool APPLY>
-__global__ void __launch_bounds__(kWarpThreads, CB_REDUCE_MIN_BLOCKS)
+constexpr int reduce_min_blocks() {
+    return GO != CB_F32 && VPL == 1 && GC > 0 && GC != 4 && !PACKED && !APPLY ? CB_REDUCE_HALF_MIN_BLOCKS
+                                                                               : CB_REDUCE_MIN_BLOCKS;
+}
+
+template <int GO, int VPL, bool PACKED, int GC, bool APPLY>
+__global__ void __launch_bounds__(kWarpThreads, reduce_min_blocks<GO, VPL, PACKED, GC, APPLY>())
     bwd_reduce_kernel(const __grid_constant__ Problem P, const __grid_constant__ Plan Q,
                       const __grid_constant__ BwdOut O, const void* grad_out, int cls) {
     if (*O.cap_fail) return;
