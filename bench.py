@@ -594,7 +594,8 @@ def run_l2_ceiling(dev, reps: int = 5):
         res[str(row_bytes)]["f16_sum_ms"] = round(ms, 4)
         del rows, rows16, idx, out
     res["how"] = ("cb_gather_ceiling: one warp per 32 random rows of an L2-resident set, 16 bytes per "
-                  "lane, 8 row steps in flight (the walkers' load shape without their bookkeeping); "
+                  "lane, 4 row steps in flight, 8 blocks of 256 threads per SM (the walkers' load shape "
+                  "without their bookkeeping, at full occupancy); "
                   "tma_*: cb_gather_ceiling_tma, four rows per TMA gather4, 8 gathers in flight per warp; "
                   "f16_sum_*: cb_gather_ceiling_f16, fp16 rows of the same size widened into fp32 sums "
                   "(the forward's 8 mixed-precision adds per 16 bytes)")

@@ -213,8 +213,10 @@ cb_status cb_tbe_sorted_payloads(const cb_tbe* h, uint32_t* out, int64_t num_ind
  * random rows out of a row set that fits in L2 (on skewed indices most rows
  * the forward gather and the backward reduce read come from L2, so this rate
  * bounds them besides the HBM bandwidth). One warp per 32 items, each lane
- * loading one 4-byte index and 16 bytes of a row per step, 8 steps in flight,
- * as those kernels load; it sums what it loads and writes one sum per 32 items.
+ * loading one 4-byte index and 16 bytes of a row per step, as those kernels
+ * load, 4 steps in flight and 8 blocks of 256 threads per SM (the rate grows
+ * with the warps resident); it sums what it loads and writes one sum per 32
+ * items.
  *   rows         device [num_rows rows of row_bytes], 16-byte aligned, read as fp32
  *   num_rows     1 .. 2^32
  *   row_bytes    64, 128, 256 or 512

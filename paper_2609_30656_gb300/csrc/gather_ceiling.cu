@@ -29,6 +29,7 @@ namespace {
 // 256 threads reach ~21 TB/s for 256-byte rows, fp32 or widened fp16, where 8
 // steps at 4-5 blocks, the register budget of the walkers, reach 15.8-20 TB/s).
 constexpr int kRows = 4;
+constexpr int kProbeBlocks = 8;  // 32 registers per thread
 
 // x's values added into acc: fp32 adds, or fp16 values widened into the fp32
 // sums by the mixed-precision add (as the forward gather adds them).
@@ -88,7 +89,7 @@ __device__ __forceinline__ float batch_sum(const uint4* __restrict__ rows, uint3
 // forward's arithmetic on half-precision tables (8 adds per 16 bytes).
 // Full batches only; the partial last batch goes to gather_tail_kernel.
 template <int G, int DT>
-__global__ void __launch_bounds__(kWarpThreads, 8) gather_ceiling_kernel(const uint4* __restrict__ rows,
+__global__ void __launch_bounds__(kWarpThreads, kProbeBlocks) gather_ceiling_kernel(const uint4* __restrict__ rows,
                                                                       int64_t num_rows,
                                                                       const uint32_t* __restrict__ idx,
                                                                       int64_t batches, float* __restrict__ out) {
