@@ -88,32 +88,46 @@ __device__ __forceinline__ int64_t run_containing(const uint32_t* seg_start, int
 // A chunk boundary at x moves to the end of the segment it falls in, unless
 // that segment is longer than the cap: short bags and runs are then never
 // split, and only heavy ones leave pieces for the fix-up. Monotone in x, so
-// consecutive chunks stay contiguous (a chunk may come out empty).
-__device__ __forceinline__ int64_t snap(const Problem& P, const Plan& Q, int mode, int t,
-                                        const uint32_t* seg_start, int64_t U, int64_t x,
-                                        int64_t p0, int64_t p1) {
-    if (Q.snap_cap <= 0 || x <= p0 || x >= p1) return x;
+// consecutive chunks stay contiguous (a chunk may come out empty). One search
+// gives both the moved boundary and the first segment of a chunk starting
+// there:
+//   mode 0: the bag touching the chunk start (the bag starting exactly there if
+//           any, the first of equal starts; else the one containing it);
+//   mode 1: the run of sorted ids containing the chunk start;
+//   mode 2: tiles only (radix sort), no moving, first left at 0.
+struct Boundary {
+    int64_t k;      // position
+    int64_t first;  // first segment of a chunk starting at k
+};
+
+__device__ __forceinline__ Boundary boundary(const Problem& P, const Plan& Q, int mode, int t,
+                                             const uint32_t* seg_start, int64_t U, int64_t x, int64_t p0,
+                                             int64_t p1) {
+    const bool may_move = Q.snap_cap > 0 && x > p0 && x < p1;
     if (mode == 0) {
-        const int64_t a = bag_lower_bound(P, t, x);
-        const int64_t bhi = static_cast<int64_t>(t) * P.B + P.B;
-        if (a > bhi) return x;
-        const int64_t e = load_index(P.offsets, a, P.is32);
-        if (e == x || a == static_cast<int64_t>(t) * P.B) return x;
-        const int64_t s0 = load_index(P.offsets, a - 1, P.is32);
-        return (e - s0 <= Q.snap_cap && e <= p1) ? e : x;
+        const int64_t blo = static_cast<int64_t>(t) * P.B, bhi = blo + P.B;
+        const int64_t a = bag_lower_bound(P, t, x);  // first bag starting at or after x
+        const int64_t e = a <= bhi ? load_index(P.offsets, a, P.is32) : -1;
+        int64_t k = x;
+        if (may_move && a <= bhi && e != x && a != blo) {
+            const int64_t s0 = load_index(P.offsets, a - 1, P.is32);
+            if (e - s0 <= Q.snap_cap && e <= p1) k = e;
+        }
+        // Moved to e (= offsets[a], with offsets[a - 1] < x < e): bag a starts
+        // there. Else the bag starting exactly at x, or the one containing it.
+        const int64_t first = (a <= bhi && e == k) ? a : a - 1;
+        return {k, min64(max64(first, blo), bhi)};
     }
     if (mode == 1) {
         const int64_t u = run_containing(seg_start, U, x);
         const int64_t s0 = seg_start[u], e = seg_start[u + 1];
-        if (s0 == x) return x;
-        return (e - s0 <= Q.snap_cap && e <= p1) ? e : x;
+        // Runs are never empty (seg_start increases), so the run containing e is u + 1.
+        if (may_move && s0 != x && e - s0 <= Q.snap_cap && e <= p1) return {e, u + 1};
+        return {x, u};
     }
-    return x;
+    return {x, 0};
 }
 
-// mode 0: first = the bag touching the chunk start (forward, key generation).
-// mode 1: first = the run of sorted ids containing the chunk start (reduce).
-// mode 2: tiles only (radix sort), first left at 0, no snapping.
 __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* seg_start,
                                    const int64_t* num_unique) {
     const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
@@ -138,25 +152,13 @@ __global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* 
         const bool last = local >= nch - 1;
         const int64_t x0 = min64(p0 + local * C, p1);
         const int64_t x1 = last ? p1 : min64(p0 + (local + 1) * C, p1);
-        const int64_t k0 = mode == 2 ? x0 : snap(P, Q, mode, t, seg_start, U, x0, p0, p1);
-        const int64_t k1 = mode == 2 || last ? x1 : snap(P, Q, mode, t, seg_start, U, x1, p0, p1);
-        const int64_t len = max64(0, k1 - k0);
-        int64_t first = 0;
-        if (mode == 0) {
-            // First bag of table t touching k0: the bag starting exactly at k0
-            // if any (the first of equal starts), else the one containing k0.
-            const int64_t blo = static_cast<int64_t>(t) * P.B, bhi = blo + P.B;
-            const int64_t a = bag_lower_bound(P, t, k0);
-            first = (a <= bhi && load_index(P.offsets, a, P.is32) == k0) ? a : a - 1;
-            first = min64(max64(first, blo), bhi);
-        } else if (mode == 1) {
-            first = run_containing(seg_start, U, k0);
-        }
+        const Boundary b0 = boundary(P, Q, mode, t, seg_start, U, x0, p0, p1);
+        const int64_t k1 = last ? x1 : boundary(P, Q, mode, t, seg_start, U, x1, p0, p1).k;
         Chunk ch;
-        ch.k0 = k0;
-        ch.first = first;
+        ch.k0 = b0.k;
+        ch.first = b0.first;
         ch.table = t;
-        ch.len = static_cast<uint32_t>(len) | (last ? 0x80000000u : 0u);
+        ch.len = static_cast<uint32_t>(max64(0, k1 - b0.k)) | (last ? 0x80000000u : 0u);
         Q.chunks[j] = ch;
     }
 }
