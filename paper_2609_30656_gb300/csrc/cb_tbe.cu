@@ -436,7 +436,7 @@ cb_status backward_impl(cb_tbe* h, int32_t batch, const void* indices, int64_t n
             S.T = h->T;
             S.segments = w.segments;
             launch_radix_pass(S, w.sp_max_tiles, stream);
-            h->launches += 4;
+            h->launches += radix_pass_launches();
         }
         cur ^= 1;
     }

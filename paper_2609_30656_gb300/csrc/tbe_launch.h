@@ -108,6 +108,7 @@ void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s);
 int radix_segments(int64_t tile_bound, int T);
 // One reduce-then-scan pass: tile counts, segment sums, slots, scatter.
 void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s);
+int radix_pass_launches();  // kernels launch_radix_pass enqueues
 
 void launch_keygen(const Problem& P, const Plan& Q, const KeyGen& K, bool packed, int64_t chunk_bound,
                    int num_sms, cudaStream_t s);

@@ -402,6 +402,73 @@ __global__ void __launch_bounds__(kRadix) radix_offsets_kernel(const SortPass S)
     }
 }
 
+// (b + c) in one kernel (CB_SORT_TABLE_SCAN): one block of 1024 threads per
+// table; thread (part, d) owns digit d over a quarter of the table's tiles.
+// It sums the part's counts (16 loads in flight), the block turns the four
+// parts' sums into each (part, digit)'s first slot (table start + the table's
+// counts of smaller digits + the earlier parts' counts of the digit), and the
+// thread replaces every count of its part by the tile's first slot. No block
+// waits on another; the per-(table, segment) blocks of (b) and (c) were
+// latency-bound on short loops.
+#ifndef CB_SORT_TABLE_SCAN
+#define CB_SORT_TABLE_SCAN 1
+#endif
+constexpr int kScanParts = 4;
+constexpr int kScanLoads = 16;
+
+__global__ void __launch_bounds__(kRadix * kScanParts) radix_table_scan_kernel(const SortPass S) {
+    __shared__ uint32_t sh_part[kScanParts][kRadix];
+    __shared__ uint32_t sh_start[kRadix];
+    __shared__ int64_t sh_scan[33];
+    const int t = blockIdx.x;
+    const int d = threadIdx.x & (kRadix - 1), part = threadIdx.x / kRadix;
+    const int64_t f = S.table_first_tile[t], e = S.table_first_tile[t + 1];
+    const int64_t per = (e - f + kScanParts - 1) / kScanParts;
+    const int64_t a = min64(f + part * per, e), b = min64(a + per, e);
+    uint32_t* c = S.tile_digits + d;
+    uint32_t sum = 0;
+    int64_t k = a;
+    for (; k + kScanLoads <= b; k += kScanLoads) {
+        uint32_t v[kScanLoads];
+#pragma unroll
+        for (int u = 0; u < kScanLoads; ++u) v[u] = c[(k + u) * kRadix];
+#pragma unroll
+        for (int u = 0; u < kScanLoads; ++u) sum += v[u];
+    }
+    for (; k < b; ++k) sum += c[k * kRadix];
+    sh_part[part][d] = sum;
+    __syncthreads();
+    uint32_t total = 0, before = 0;
+#pragma unroll
+    for (int q = 0; q < kScanParts; ++q) {
+        const uint32_t x = sh_part[q][d];
+        before += q < part ? x : 0u;
+        total += x;
+    }
+    // digit starts: the scan over the first part's threads (0..255, one per digit)
+    int64_t all;
+    const int64_t ex = block_excl_scan(part == 0 ? total : 0u, sh_scan, &all);
+    // positions are below 2^30: 32 bits hold every slot
+    if (part == 0) sh_start[d] = static_cast<uint32_t>(S.table_pos[t] + ex);
+    __syncthreads();
+    uint32_t run = sh_start[d] + before;
+    for (k = a; k + kScanLoads <= b; k += kScanLoads) {
+        uint32_t v[kScanLoads];
+#pragma unroll
+        for (int u = 0; u < kScanLoads; ++u) v[u] = c[(k + u) * kRadix];
+#pragma unroll
+        for (int u = 0; u < kScanLoads; ++u) {
+            c[(k + u) * kRadix] = run;
+            run += v[u];
+        }
+    }
+    for (; k < b; ++k) {
+        const uint32_t v = c[k * kRadix];
+        c[k * kRadix] = run;
+        run += v;
+    }
+}
+
 // (d) The scatter of tile blockIdx.x: the ranking of the single-sweep kernel,
 // with the first output slot of every digit read from (c). NT threads per tile
 // (NT / 32 warps ranking kSortTile / NT keys per thread); threads 0..255 own one
@@ -556,8 +623,12 @@ void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     const unsigned grid = static_cast<unsigned>(max64(tile_bound, 1));
     const unsigned parts = static_cast<unsigned>(S.T) * static_cast<unsigned>(S.segments);
     radix_count_kernel<<<grid, kSortThreads, 0, s>>>(S);
-    radix_segsum_kernel<<<parts, kRadix, 0, s>>>(S);
-    radix_offsets_kernel<<<parts, kRadix, 0, s>>>(S);
+    if (CB_SORT_TABLE_SCAN) {
+        radix_table_scan_kernel<<<static_cast<unsigned>(S.T), kRadix * kScanParts, 0, s>>>(S);
+    } else {
+        radix_segsum_kernel<<<parts, kRadix, 0, s>>>(S);
+        radix_offsets_kernel<<<parts, kRadix, 0, s>>>(S);
+    }
     static bool configured = false;
     if (!configured) {  // static + dynamic shared memory may pass the 48 KB default
         cudaFuncSetAttribute(radix_scatter_kernel<kScatterThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -566,6 +637,8 @@ void launch_radix_pass(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     }
     radix_scatter_kernel<kScatterThreads><<<grid, kScatterThreads, kSortDynSmem, s>>>(S);
 }
+
+int radix_pass_launches() { return CB_SORT_TABLE_SCAN ? 3 : 4; }
 
 void launch_onesweep(const SortPass& S, int64_t tile_bound, cudaStream_t s) {
     static bool configured = false;
