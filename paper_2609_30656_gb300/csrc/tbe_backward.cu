@@ -222,23 +222,35 @@ __global__ void __launch_bounds__(kRleThreads) rle_count_kernel(const uint32_t* 
     if (threadIdx.x == 0) tile_heads[blockIdx.x] = total;
 }
 
-// One block: thread i sums a contiguous range of the tile counts, one block
-// scan, then the thread writes its range's exclusive prefixes.
+// One block over the tile counts in rounds of 1024 x 8: thread i takes 8
+// consecutive counts of the round (a warp reads 2 KB contiguous), one block
+// scan per round, the round's total carried into the next: 45 us on cfg5.
+// (With each thread owning 1/1024 of the counts every warp load touched 32
+// lines: 55 us; with 16 counts per thread, at 64 registers: 57 us.)
 __global__ void __launch_bounds__(1024) rle_scan_kernel(const int64_t* tile_heads, int64_t tiles,
                                                         int64_t* tile_base, int64_t* num_unique) {
+    constexpr int kPer = 8;
     __shared__ int64_t sh[33];
-    const int64_t per = (tiles + blockDim.x - 1) / blockDim.x;
-    const int64_t lo = min64(static_cast<int64_t>(threadIdx.x) * per, tiles), hi = min64(lo + per, tiles);
-    int64_t sum = 0;
-    for (int64_t i = lo; i < hi; ++i) sum += tile_heads[i];
-    int64_t total;
-    int64_t run = block_excl_scan(sum, sh, &total);
-    for (int64_t i = lo; i < hi; ++i) {
-        const int64_t c = tile_heads[i];
-        tile_base[i] = run;
-        run += c;
+    int64_t carry = 0;
+    for (int64_t c0 = 0; c0 < tiles; c0 += static_cast<int64_t>(blockDim.x) * kPer) {
+        const int64_t i0 = c0 + static_cast<int64_t>(threadIdx.x) * kPer;
+        int64_t v[kPer];
+        int64_t sum = 0;
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) {
+            v[u] = i0 + u < tiles ? tile_heads[i0 + u] : 0;
+            sum += v[u];
+        }
+        int64_t total;
+        int64_t run = carry + block_excl_scan(sum, sh, &total);
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) {
+            if (i0 + u < tiles) tile_base[i0 + u] = run;
+            run += v[u];
+        }
+        carry += total;
     }
-    if (threadIdx.x == 0) *num_unique = total;
+    if (threadIdx.x == 0) *num_unique = carry;
 }
 
 // Each warp writes its run heads (unique key, start position) 32 at a time,
