@@ -113,8 +113,15 @@ __device__ __forceinline__ bool bags_by_mask(const BagWindow32& W, int32_t p0, i
 #endif
 constexpr int kKeygenSteps = CB_KEYGEN_STEPS;
 
+// Resident blocks per SM the unpacked key generation is compiled for: 6 (40
+// registers) against the 5 its registers gave unbounded: cfg5 0.748 -> 0.677 ms,
+// cfg5u 0.748 -> 0.636 ms on one box. The packed form (80 registers) keeps its own.
+#ifndef CB_KEYGEN_MIN_BLOCKS
+#define CB_KEYGEN_MIN_BLOCKS 6
+#endif
 template <bool PACKED>
-__global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q, KeyGen K) {
+__global__ void __launch_bounds__(kWarpThreads, PACKED ? 1 : CB_KEYGEN_MIN_BLOCKS)
+    keygen_kernel(Problem P, Plan Q, KeyGen K) {
     const int lane = threadIdx.x & 31;
     const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     // all classes' chunks in one sequence: the counter after the classes' own
