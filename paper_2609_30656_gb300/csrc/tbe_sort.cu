@@ -313,7 +313,10 @@ __global__ void __launch_bounds__(kSortThreads, 3) onesweep_kernel(SortPass S) {
 
 // (a) Digit counts of every tile of this pass: 16 keys per thread, shared
 // counters (their order does not matter here).
-__global__ void __launch_bounds__(kSortThreads) radix_count_kernel(const SortPass S) {
+#ifndef CB_COUNT_MIN_BLOCKS
+#define CB_COUNT_MIN_BLOCKS 8  // resident blocks per SM the count kernel is compiled for (31 registers)
+#endif
+__global__ void __launch_bounds__(kSortThreads, CB_COUNT_MIN_BLOCKS) radix_count_kernel(const SortPass S) {
     __shared__ uint32_t sh[kRadix];
     const int64_t tile = blockIdx.x;
     if (tile >= *S.num_tiles) return;  // the grid is an upper bound on the tiles
