@@ -128,8 +128,11 @@ __device__ __forceinline__ Boundary boundary(const Problem& P, const Plan& Q, in
     return {x, 0};
 }
 
-__global__ void plan_chunks_kernel(Problem P, Plan Q, int mode, const uint32_t* seg_start,
-                                   const int64_t* num_unique) {
+// 8 blocks of 256 threads per SM (32 registers): the grid (8 per SM) runs in
+// one wave of latency-bound searches.
+__global__ void __launch_bounds__(256, 8) plan_chunks_kernel(Problem P, Plan Q, int mode,
+                                                             const uint32_t* seg_start,
+                                                             const int64_t* num_unique) {
     const int64_t total = min64(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     const int64_t C = Q.chunk_len;
