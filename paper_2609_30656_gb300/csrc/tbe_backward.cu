@@ -113,11 +113,11 @@ __device__ __forceinline__ bool bags_by_mask(const BagWindow32& W, int32_t p0, i
 #endif
 constexpr int kKeygenSteps = CB_KEYGEN_STEPS;
 
-// Resident blocks per SM the unpacked key generation is compiled for: 6 (40
-// registers) against the 5 its registers gave unbounded: cfg5 0.748 -> 0.677 ms,
-// cfg5u 0.748 -> 0.636 ms on one box. The packed form (80 registers) keeps its own.
+// Resident blocks per SM the unpacked key generation is compiled for (1: as
+// its registers allow, 5 blocks at 48). 6 blocks (40 registers) was faster on
+// one box and slower on uniform indices on two others (cfg5u 0.626 -> 0.711 ms).
 #ifndef CB_KEYGEN_MIN_BLOCKS
-#define CB_KEYGEN_MIN_BLOCKS 6
+#define CB_KEYGEN_MIN_BLOCKS 1
 #endif
 template <bool PACKED>
 __global__ void __launch_bounds__(kWarpThreads, PACKED ? 1 : CB_KEYGEN_MIN_BLOCKS)
