@@ -10,6 +10,14 @@
 #include "tbe_internal.cuh"
 #include "tbe_launch.h"
 
+// The reduce with the optimizer step fused carries more state (the table row
+// and its update), so it spilled at 3 blocks with 8 rows; measured on cfg5
+// (fused SGD / Adagrad ms): 8 rows at 3 blocks 14.46 / 17.24, 4 at 4 13.25 /
+// 15.47, 4 at 5 13.00 / 15.05, 2 at 5 12.93 / 14.83, 2 at 6 13.22 / 14.88,
+// 1 at 5 13.73 / 15.67.
+#ifndef CB_REDUCE_APPLY_ROWS
+#define CB_REDUCE_APPLY_ROWS 2  // rows in flight per lane with the optimizer step fused
+#endif
 #ifndef CB_REDUCE_HALF_ROWS
 #define CB_REDUCE_HALF_ROWS 4  // rows in flight per lane for fp16 / bf16 grad_out
 #endif
@@ -160,7 +168,7 @@ struct BwdPolicy {
     // Half grad_out rows (8 values per lane, usually 2 rows per warp step) take
     // the forward's code shape: fewer rows in flight, one copy of the run-end
     // code per batch.
-    static constexpr int kRows = GO == CB_F32 ? CB_REDUCE_ROWS : CB_REDUCE_HALF_ROWS;
+    static constexpr int kRows = APPLY ? CB_REDUCE_APPLY_ROWS : (GO == CB_F32 ? CB_REDUCE_ROWS : CB_REDUCE_HALF_ROWS);
     static constexpr int kUnroll = kRows / VPL > 0 ? kRows / VPL : 1;
     static constexpr bool kWeighted = PACKED;
     static constexpr bool kUnrollGroups = GO == CB_F32 ? CB_REDUCE_UNROLL_GROUPS : false;
@@ -274,10 +282,14 @@ struct BwdPolicy {
 #ifndef CB_REDUCE_HALF_MIN_BLOCKS
 #define CB_REDUCE_HALF_MIN_BLOCKS 5
 #endif
+#ifndef CB_REDUCE_APPLY_MIN_BLOCKS
+#define CB_REDUCE_APPLY_MIN_BLOCKS 5  // the reduce with the optimizer step fused
+#endif
 template <int GO, int VPL, bool PACKED, int GC, bool APPLY>
 constexpr int reduce_min_blocks() {
-    return GO != CB_F32 && VPL == 1 && GC > 0 && GC != 4 && !PACKED && !APPLY ? CB_REDUCE_HALF_MIN_BLOCKS
-                                                                               : CB_REDUCE_MIN_BLOCKS;
+    if (APPLY) return CB_REDUCE_APPLY_MIN_BLOCKS;
+    return GO != CB_F32 && VPL == 1 && GC > 0 && GC != 4 && !PACKED ? CB_REDUCE_HALF_MIN_BLOCKS
+                                                                    : CB_REDUCE_MIN_BLOCKS;
 }
 
 template <int GO, int VPL, bool PACKED, int GC, bool APPLY>
