@@ -113,15 +113,11 @@ __device__ __forceinline__ bool bags_by_mask(const BagWindow32& W, int32_t p0, i
 #endif
 constexpr int kKeygenSteps = CB_KEYGEN_STEPS;
 
-// Resident blocks per SM the unpacked key generation is compiled for (1: as
-// its registers allow, 5 blocks at 48). 6 blocks (40 registers) was faster on
-// one box and slower on uniform indices on two others (cfg5u 0.626 -> 0.711 ms).
-#ifndef CB_KEYGEN_MIN_BLOCKS
-#define CB_KEYGEN_MIN_BLOCKS 1
-#endif
+// Compiled with no minimum of resident blocks: 48 registers, 5 blocks of 256
+// threads per SM. (A minimum of 1 let it take 72 registers, 3 blocks: cfg5
+// 0.63 -> 0.75 ms; a minimum of 6, 40 registers: cfg5u 0.63 -> 0.71 ms.)
 template <bool PACKED>
-__global__ void __launch_bounds__(kWarpThreads, PACKED ? 1 : CB_KEYGEN_MIN_BLOCKS)
-    keygen_kernel(Problem P, Plan Q, KeyGen K) {
+__global__ void __launch_bounds__(kWarpThreads) keygen_kernel(Problem P, Plan Q, KeyGen K) {
     const int lane = threadIdx.x & 31;
     const int64_t total = min(Q.class_chunk_base[Q.num_classes], Q.max_chunks);
     // all classes' chunks in one sequence: the counter after the classes' own
