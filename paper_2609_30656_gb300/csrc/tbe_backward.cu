@@ -256,6 +256,10 @@ __global__ void __launch_bounds__(1024) rle_scan_kernel(const int64_t* tile_head
     if (threadIdx.x == 0) *num_unique = carry;
 }
 
+#ifndef CB_RLE_FNS
+#define CB_RLE_FNS 1  // find a lane's n-th head with __fns (0: clear the earlier heads one by one)
+#endif
+
 // Each warp writes its run heads (unique key, start position) 32 at a time,
 // coalesced: lane l writes the warp's head x = x0 + l, found by a search over
 // the lanes' head prefixes (the owning lane) and then among that lane's 16 head
@@ -286,8 +290,15 @@ __global__ void __launch_bounds__(kRleThreads) rle_write_kernel(const uint32_t* 
         uint32_t f = __shfl_sync(kFull, flags, j);
         const int32_t mj = __shfl_sync(kFull, mine, j);
         if (x < wtot) {
-            for (int32_t r = x - mj; r > 0; --r) f &= f - 1;  // drop the lane's earlier heads
-            const int64_t pos = wbase + static_cast<int64_t>(j) * kRleItems + (__ffs(f) - 1);
+            // head x is the lane's (x - mj + 1)-th head: that set bit of its flags
+            int bit;
+            if (CB_RLE_FNS) {
+                bit = static_cast<int>(__fns(f, 0, x - mj + 1));
+            } else {
+                for (int32_t r = x - mj; r > 0; --r) f &= f - 1;  // drop the lane's earlier heads
+                bit = __ffs(f) - 1;
+            }
+            const int64_t pos = wbase + static_cast<int64_t>(j) * kRleItems + bit;
             uo[x] = __ldg(keys + pos);
             so[x] = static_cast<uint32_t>(pos);
         }
