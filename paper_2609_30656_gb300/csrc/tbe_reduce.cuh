@@ -277,8 +277,10 @@ struct BwdPolicy {
 // Resident blocks per SM the reduce is compiled for: half-precision grad_out
 // slices with one vector per lane, no coefficient and no optimizer step fit 5
 // blocks' registers (48) without spilling, and more resident warps raise the
-// rate of the L2-served gathers; fp32 slices (8 rows in flight per lane) and
-// the other forms keep CB_REDUCE_MIN_BLOCKS.
+// rate of the L2-served gathers; the optimizer-step form runs 5 blocks with
+// 2 rows in flight (CB_REDUCE_APPLY_ROWS); fp32 slices (8 rows in flight per
+// lane, whose uniform-index gathers come from DRAM and want the bytes in
+// flight) and the other forms keep CB_REDUCE_MIN_BLOCKS.
 #ifndef CB_REDUCE_HALF_MIN_BLOCKS
 #define CB_REDUCE_HALF_MIN_BLOCKS 5
 #endif
