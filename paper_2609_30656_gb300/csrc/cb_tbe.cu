@@ -16,8 +16,14 @@ using namespace cbtbe;
 
 namespace {
 
-constexpr int64_t kFwdChunk = 512;   // lookups per forward chunk
-constexpr int64_t kBwdChunk = 512;   // sorted positions per reduce chunk
+#ifndef CB_FWD_CHUNK
+#define CB_FWD_CHUNK 512
+#endif
+#ifndef CB_BWD_CHUNK
+#define CB_BWD_CHUNK 512
+#endif
+constexpr int64_t kFwdChunk = CB_FWD_CHUNK;  // lookups per forward chunk
+constexpr int64_t kBwdChunk = CB_BWD_CHUNK;  // sorted positions per reduce chunk
 constexpr uint64_t kLookbackTimeoutNs = 1000000000ull;  // 1 s bounded wait
 constexpr int kNumTimers = 7;
 const char* const kComponentNames[kNumTimers] = {"fwd.prep",   "fwd.gather", "fwd.fixup",
